@@ -1,0 +1,6 @@
+"""Seeded synthetic inputs shared by the oracle tests, the CUDA tests and the benchmark.
+
+Holds input generation only; no part of the sparse product is computed here.
+"""
+from .matrices import *  # noqa: F401,F403
+from .matrices import HostCSR, WORKLOADS, WORKLOAD_ORDER, row_subset, workload  # noqa: F401
