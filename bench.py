@@ -1,0 +1,383 @@
+"""Benchmark of C = A*B (CSR SpGEMM) on the GPU, one JSON line on stdout.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+A step is one full product -- symbolic pass (including its nnz read-back),
+allocation of C, numeric pass and the final status read -- over device-
+resident inputs.  Between timed steps the L2 is flushed by writing a buffer
+larger than it; each step is timed with CUDA events on the stream the
+library runs on.  Throughput is GFLOP/s = 2 x products / time; the
+effective HBM bandwidth uses the compulsory bytes (read A and B once, write
+C once, at their stored widths).
+
+Extra keys: `e2e` (the same product through the public Python API from
+pinned host inputs to the host copy of C, copies inside the timed region),
+`roofline` (the numeric pass, the dominant launch, against the measured
+copy bandwidth), `cpu_baseline` (the CPU oracle on a bounded row sample, on
+this host's cores), `clocks` (nvidia-smi samples during the timed region).
+
+Under torchrun (N > 1) every rank runs its own replica of the workload on its
+own GPU (no collective on the data path); rank 0 prints the line with the
+maximum time over ranks.  `--impl reference` times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from synth import WORKLOADS, workload  # noqa: E402
+
+METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per config"
+DEFAULT_WORKLOAD = "uniform_rect_1m"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def products_per_row(A, B) -> np.ndarray:
+    lenB = np.diff(B.rowptr)
+    ub = np.zeros(A.nrows, dtype=np.int64)
+    if A.nnz:
+        np.add.at(ub, np.repeat(np.arange(A.nrows), np.diff(A.rowptr)), lenB[A.colidx])
+    return ub
+
+
+def csr_bytes(nrows: int, nnz: int, value_bytes: int) -> int:
+    return 8 * (nrows + 1) + (4 + value_bytes) * nnz
+
+
+def measured_peaks() -> dict:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            d = json.load(fh)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines: list[str] = []
+        self._t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return self
+        self._t = threading.Thread(target=self._read, daemon=True)
+        self._t.start()
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict | None:
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self._t:
+            self._t.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline(A, B, ub: np.ndarray, target_s: float, seed: int = 0) -> dict:
+    """The CPU oracle on a seeded row sample sized to about target_s seconds."""
+    from oracle import oracle_spgemm
+    cores = os.cpu_count() or 1
+    rng = np.random.default_rng(seed)
+    probe = np.sort(rng.choice(A.nrows, size=min(A.nrows, 512), replace=False))
+    t0 = time.perf_counter()
+    oracle_spgemm(A, B, rows=probe, threads=cores)
+    dt = max(time.perf_counter() - t0, 1e-6)
+    per_product = dt / max(int(ub[probe].sum()), 1)
+    want_products = target_s / per_product
+    nrows = int(min(A.nrows, max(probe.size, want_products / max(ub.mean(), 1e-9))))
+    rows = np.sort(rng.choice(A.nrows, size=nrows, replace=False))
+    t0 = time.perf_counter()
+    oracle_spgemm(A, B, rows=rows, threads=cores)
+    dt = time.perf_counter() - t0
+    prods = int(ub[rows].sum())
+    return {"value": round(2.0 * prods / dt / 1e9, 4), "unit": "GFLOP/s", "cores": cores, "kind": "oracle",
+            "sample": f"{nrows} of {A.nrows} rows (seeded uniform sample, {prods} products), "
+                      f"{dt:.1f} s, std::map per row, {cores} threads"}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+        pg = dist
+    return world, rank, local, pg
+
+
+def reduce_max(x: float, world: int, pg, device) -> float:
+    if world == 1:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int, pg) -> None:
+    if world > 1:
+        pg.barrier()
+
+
+def run_reference(args, world, rank) -> None:
+    """CPU oracle arm: each step computes a bounded row sample on the host cores."""
+    if rank != 0:
+        return
+    from oracle import oracle_spgemm
+    A, B = workload(args.workload)
+    ub = products_per_row(A, B)
+    cores = os.cpu_count() or 1
+    rng = np.random.default_rng(1234)
+    # size one step to about args.ref_step_s seconds
+    probe = np.sort(rng.choice(A.nrows, size=min(A.nrows, 512), replace=False))
+    t0 = time.perf_counter()
+    oracle_spgemm(A, B, rows=probe, threads=cores)
+    per_product = max(time.perf_counter() - t0, 1e-6) / max(int(ub[probe].sum()), 1)
+    nrows = int(min(A.nrows, max(probe.size, args.ref_step_s / per_product / max(ub.mean(), 1e-9))))
+    rows = np.sort(rng.choice(A.nrows, size=nrows, replace=False))
+    prods = int(ub[rows].sum())
+    for _ in range(args.warmup):
+        oracle_spgemm(A, B, rows=rows, threads=cores)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_spgemm(A, B, rows=rows, threads=cores)
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = 2.0 * prods * args.steps / total / 1e9
+    sample = f"{nrows} of {A.nrows} rows per step (seeded uniform sample, {prods} products), {cores} threads"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GFLOP/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": str(A.vals.dtype).replace("float", "f"),
+        "data": "synthetic", "config": {"workload": args.workload, "description": WORKLOADS[args.workload]},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GFLOP/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, world, rank, local, pg) -> None:
+    import torch
+    from paper_2606_20855_gb300 import _abi
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+
+    _abi.load()
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    A, B = workload(args.workload)
+    same = B is A
+    ub = products_per_row(A, B)
+    products = int(ub.sum())
+    s = 8 if A.vals.dtype == np.float64 else 4
+    stream = torch.cuda.current_stream(device)
+
+    dA = DeviceCSR.from_host(A, device)
+    dB = dA if same else DeviceCSR.from_host(B, device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
+
+    op = SpGEMM(dA, dB)
+    out = None
+
+    def step():
+        nonlocal out
+        op.symbolic()
+        out = op.numeric(out)
+        op.wait()
+
+    for _ in range(args.warmup):
+        step()
+    nnz = op.nnz
+    info = op.plan_info()
+    algo_bytes = csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz, s)
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local).start() if rank == 0 else None
+    barrier(world, pg)
+    torch.cuda.synchronize(device)
+    for i in range(args.steps):
+        flush.fill_(i)  # write > L2 between timed steps (not timed)
+        e0, e1, e2 = ev[i]
+        e0.record(stream)
+        op.symbolic()
+        e1.record(stream)
+        out = op.numeric(out)
+        e2.record(stream)
+        op.wait()
+    torch.cuda.synchronize(device)
+    barrier(world, pg)
+    clk = clocks.stop() if clocks else None
+    step_ms = [a.elapsed_time(c) for a, _, c in ev]
+    num_ms = [b.elapsed_time(c) for _, b, c in ev]
+    sym_ms = [a.elapsed_time(b) for a, b, _ in ev]
+    total_s = sum(step_ms) / 1e3
+    total_s = reduce_max(total_s, world, pg, device)
+    launches_per_step = info["symbolic_launches"] + info["numeric_launches"]
+
+    # End to end through the public API: pinned host inputs -> device -> product -> host C.
+    e2e = None
+    if args.e2e_steps > 0:
+        hA = [torch.from_numpy(a).pin_memory() for a in (A.rowptr, A.colidx, A.vals)]
+        hB = hA if same else [torch.from_numpy(a).pin_memory() for a in (B.rowptr, B.colidx, B.vals)]
+        h_col = torch.empty(nnz, dtype=torch.int32).pin_memory()
+        h_val = torch.empty(nnz, dtype=hA[2].dtype).pin_memory()
+        h_rp = torch.empty(A.nrows + 1, dtype=torch.int64).pin_memory()
+
+        def e2e_step():
+            tA = DeviceCSR(A.nrows, A.ncols, *[t.to(device, non_blocking=True) for t in hA])
+            tB = tA if same else DeviceCSR(B.nrows, B.ncols, *[t.to(device, non_blocking=True) for t in hB])
+            with SpGEMM(tA, tB) as op2:
+                op2.symbolic()
+                C = op2.numeric()
+                h_rp.copy_(C.rowptr, non_blocking=True)
+                h_col.copy_(C.colidx, non_blocking=True)
+                h_val.copy_(C.vals, non_blocking=True)
+                op2.wait()
+            torch.cuda.synchronize(device)
+
+        e2e_step()
+        barrier(world, pg)
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2e_s = reduce_max(time.perf_counter() - t0, world, pg, device)
+        h2d = sum(t.numel() * t.element_size() for t in hA) + (0 if same else sum(t.numel() * t.element_size() for t in hB))
+        d2h = h_rp.numel() * 8 + h_col.numel() * 4 + h_val.numel() * h_val.element_size()
+        e2e = {"value": round(2.0 * products * args.e2e_steps * world / e2e_s / 1e9, 3), "unit": "GFLOP/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
+
+    op.close()
+    if rank != 0:
+        return
+    peaks = measured_peaks()
+    num_mean_s = statistics.mean(num_ms) / 1e3
+    num_achieved = algo_bytes / num_mean_s / 1e9
+    value = 2.0 * products * args.steps * world / total_s / 1e9
+    eff_gbs = algo_bytes * args.steps * world / total_s / 1e9
+    base = None
+    if args.cpu_baseline_s > 0:
+        base = cpu_baseline(A, B, ub, args.cpu_baseline_s)
+    line = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": "GFLOP/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(1e3 * total_s / args.steps, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64" if s == 8 else "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": args.workload, "description": WORKLOADS[args.workload],
+            "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_a": A.nnz, "nnz_b": B.nnz, "nnz_c": int(nnz),
+            "products": products, "l2": "flushed between timed steps (write of a buffer > L2)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        },
+        "effective_hbm_gbs": round(eff_gbs, 1),
+        "frac_of_8tbs": round(eff_gbs / NOMINAL_HBM_GBS, 4),
+        "phases_ms": {"symbolic_median": round(statistics.median(sym_ms), 4),
+                      "numeric_median": round(statistics.median(num_ms), 4),
+                      "step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
+        "roofline": {
+            "kernel": "numeric pass (hash-bin rows)", "bound": "hbm", "achieved": round(num_achieved, 1),
+            "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(num_achieved / peaks["hbm_gbs"], 4),
+            "peak_source": peaks["source"], "traffic": args.traffic,
+        },
+        "gpu_launches": int(launches_per_step * args.steps),
+        "plan": info,
+        "clocks": clk,
+        "e2e": e2e,
+        "cpu_baseline": base,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None) -> int:
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=list(WORKLOADS), default=DEFAULT_WORKLOAD)
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
+    ap.add_argument("--ref-step-s", type=float, default=4.0, help="seconds per reference-arm step")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="ncu DRAM bytes per numeric launch, when captured for the current kernels")
+    args = ap.parse_args(argv)
+    world, rank, local, pg = dist_setup()
+    try:
+        if args.impl == "reference":
+            run_reference(args, world, rank)
+        else:
+            run_ours(args, world, rank, local, pg)
+    finally:
+        if pg is not None:
+            pg.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,180 @@
+/*
+ * ws_spgemm.h -- C ABI of the GB300 (sm_103a) sparse x sparse -> sparse
+ * matrix multiply, C = A * B, with A, B and C in CSR.
+ *
+ * The operation is the sparse product whose parallel form is Gustavson's
+ * algorithm (Sec. 5.1, Fig. "SpGEMM implemented in WingSpan"): every output
+ * row C[i,:] = sum over stored A[i,k] of A[i,k] * B[k,:] is owned by exactly
+ * one worker, which accumulates it in a private workspace and then writes its
+ * own, disjoint segment of C (the shard level of Sec. 4, used for SpGEMM in
+ * Sec. 5.1).  The output must satisfy the compressed-format invariants the
+ * paper singles out (Sec. 1 and Sec. 3.1: monotone prefix-sum position
+ * arrays over contiguous buffers).  The calls follow the tensor lifecycle of
+ * Sec. 4 (declare -> update -> freeze): a symbolic pass sizes C and fills its
+ * row pointer, the caller allocates C's index and value arrays, and a numeric
+ * pass fills them.
+ *
+ * CSR layout used by every call (0-based):
+ *   rowptr  int64_t[nrows + 1], rowptr[0] = 0, non-decreasing, rowptr[nrows] = nnz
+ *   colidx  int32_t[nnz], strictly increasing within each row, in [0, ncols)
+ *   vals    float[nnz] or double[nnz] (ws_dtype_t)
+ * All array pointers are DEVICE pointers on the current CUDA device and are
+ * borrowed: the library never frees them, and the caller keeps them alive
+ * until the last call that uses the handle has completed on its stream.
+ *
+ * Result semantics:
+ *   - structure: C holds (i, j) iff some stored A[i,k] meets a stored B[k,j]
+ *     (structural product; an entry whose sum is exactly zero is kept, stored
+ *     zeros in A or B count as entries);
+ *   - column indices of every row of C are strictly increasing;
+ *   - values are accumulated in the value type of A and B; the order of the
+ *     additions is unspecified (results agree with an ordered sequential sum
+ *     up to rounding).
+ *
+ * Errors: every call returns a ws_status_t; no call throws or aborts.
+ * Argument, shape and dtype errors are detected on the host before any work
+ * is queued.  Failures detected by a kernel are recorded in a status word
+ * that the library reads at its next synchronisation point (the end of
+ * ws_spgemm_symbolic, or ws_spgemm_wait).  Kernels never trap and every
+ * device loop is bounded.  ws_last_error() gives a one-line description of
+ * the most recent failure on the calling thread.
+ *
+ * Threading: handles are not thread-safe.  One output handle serves one
+ * product at a time; use separate output handles for products that run
+ * concurrently.
+ */
+#ifndef WS_SPGEMM_H
+#define WS_SPGEMM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* ws_stream_t;
+
+typedef struct ws_csr_s* ws_csr_t;
+
+typedef enum {
+  WS_F32 = 1, /* float  */
+  WS_F64 = 2  /* double */
+} ws_dtype_t;
+
+typedef enum {
+  WS_OK = 0,
+  WS_ERR_INVALID_ARG = 1, /* NULL handle/pointer, negative size, bad enum        */
+  WS_ERR_INVALID_CSR = 2, /* validation found broken CSR invariants              */
+  WS_ERR_SHAPE = 3,       /* A.ncols != B.nrows, or C is not A.nrows x B.ncols     */
+  WS_ERR_DTYPE = 4,       /* A, B and C do not share one value type              */
+  WS_ERR_OVERFLOW = 5,    /* a size exceeds what the index types can hold         */
+  WS_ERR_ALLOC = 6,       /* device or pinned-host allocation failed             */
+  WS_ERR_CUDA = 7,        /* a CUDA runtime call failed                          */
+  WS_ERR_DEVICE = 8,      /* a kernel gave up (bounded loop ran out) -- internal  */
+  WS_ERR_STATE = 9        /* calls out of order (numeric before symbolic, ...)   */
+} ws_status_t;
+
+/*
+ * ws_csr_create -- wraps borrowed device CSR arrays in a handle.
+ *   out      receives the handle (set to NULL on failure)
+ *   nrows, ncols  matrix shape, 0 <= nrows, 0 <= ncols <= INT32_MAX
+ *   nnz      number of stored entries (ignored for an output handle, pass 0)
+ *   rowptr   int64[nrows + 1] device array (required, also for C: the
+ *            symbolic pass writes C's row pointer into it)
+ *   colidx   int32[nnz] device array; may be NULL when nnz == 0 or for an
+ *            output handle before ws_spgemm_numeric
+ *   vals     value array of type dtype; same NULL rule as colidx
+ *   dtype    WS_F32 or WS_F64
+ *   validate non-zero: check the CSR invariants listed above on the device
+ *            (O(nrows + nnz) work, synchronises `stream`); a violation gives
+ *            WS_ERR_INVALID_CSR and no handle.  Pass 0 for an output handle.
+ *   stream   stream for the validation kernel
+ * The handle owns only library scratch (released by ws_csr_destroy).
+ */
+ws_status_t ws_csr_create(ws_csr_t* out, int64_t nrows, int64_t ncols, int64_t nnz, int64_t* rowptr,
+                          int32_t* colidx, void* vals, ws_dtype_t dtype, int validate,
+                          ws_stream_t stream);
+
+/*
+ * ws_spgemm_symbolic -- structure pass of C = A * B.
+ * Computes, for every row i, the number of distinct columns of
+ * sum_k A[i,k] B[k,:], writes C.rowptr (exclusive prefix sum, C.rowptr[0] = 0)
+ * into the rowptr array given to C's handle, and returns nnz(C) in *nnz_out
+ * (host pointer).  C must be an output handle of shape A.nrows x B.ncols and
+ * the same dtype.  Work is queued on `stream`; the call returns after the
+ * stream has reached the end of the pass (it synchronises `stream`), because
+ * the caller needs nnz(C) to allocate C's arrays.  The row plan (row classes,
+ * per-row workspaces) is kept in C's handle for ws_spgemm_numeric.
+ * Device scratch is allocated stream-ordered on `stream` and cached in C's
+ * handle across calls.
+ */
+ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_out, ws_stream_t stream);
+
+/*
+ * ws_spgemm_numeric -- value pass of C = A * B.
+ *   c_colidx  device int32[nnz(C)] written with C's column indices
+ *   c_vals    device value array [nnz(C)] of C's dtype
+ * Requires a completed ws_spgemm_symbolic for the same A, B and C (and A, B
+ * unchanged since).  Asynchronous: work is queued on `stream` and the call
+ * returns without waiting; device-side failures are reported by
+ * ws_spgemm_wait.  The two arrays are recorded in C's handle.
+ */
+ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                              ws_stream_t stream);
+
+/*
+ * ws_spgemm_wait -- synchronises `stream` and returns the device status
+ * recorded by the last symbolic/numeric pass of C (WS_OK if none failed).
+ */
+ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream);
+
+/*
+ * ws_csr_destroy -- releases the handle and the scratch it owns (never the
+ * borrowed arrays).  NULL-safe.  Synchronises the device if the handle owns
+ * scratch, so pending work that uses it completes first.
+ */
+ws_status_t ws_csr_destroy(ws_csr_t handle);
+
+/* Short static description of a status code. */
+const char* ws_status_string(ws_status_t status);
+
+/* One-line description of the most recent failure on the calling thread ("" if none). */
+const char* ws_last_error(void);
+
+/*
+ * ws_csr_nnz -- number of entries of a handle (for C: nnz(C) after symbolic,
+ * -1 before).  Returns WS_ERR_INVALID_ARG for a NULL handle or pointer.
+ */
+ws_status_t ws_csr_nnz(ws_csr_t handle, int64_t* nnz_out);
+
+/*
+ * ws_spgemm_plan_info -- counts from the last symbolic pass of C, for
+ * diagnostics and tests: info[0] empty rows, info[1] single-entry (direct
+ * copy) rows, info[2] hash rows, info[3] hash rows re-routed to the sorting
+ * path, info[4] dense-window rows, info[5] dense-window slices,
+ * info[6] total products (sum over rows of the product count),
+ * info[7] number of kernel launches queued by the last symbolic pass,
+ * info[8] number queued by the last numeric pass.
+ * `n` is the length of `info` (at most 9 values are written).
+ */
+ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
+
+/*
+ * ws_set_tuning -- test/diagnostic knob, process-wide.
+ *   key 1: largest product count of a row that uses the shared-memory hash
+ *          path (default 4096; smaller values send more rows to the
+ *          dense-window path, 0 sends every multi-entry row there)
+ *   key 2: longest run of occupied hash slots the sort-free ranking accepts
+ *          (default 64; smaller values send more rows to the sorting path)
+ *   key 3: dense-window slice width in columns (default 8192 for double,
+ *          16384 for float; must be a multiple of 1024, 0 = default)
+ * Returns WS_ERR_INVALID_ARG for an unknown key or out-of-range value.
+ */
+ws_status_t ws_set_tuning(int key, int64_t value);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WS_SPGEMM_H */

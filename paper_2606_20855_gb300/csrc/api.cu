@@ -1,0 +1,529 @@
+// C ABI of the SpGEMM library (declared in include/ws_spgemm.h).
+//
+// Symbolic pass (ws_spgemm_symbolic), all on the caller's stream:
+//   1. analyze   per-row product count, column range, class       (2 launches)
+//   -- read the class counts back (one small copy + stream sync)
+//   2. scatter   group rows by class                                (1 launch)
+//   3. dense     expand dense-window rows into column slices, count (2 launches)
+//   4. hash      count distinct columns per hash bin                (1 launch per non-empty bin)
+//   5. scan      counts -> C.rowptr                                 (3 launches)
+//   -- read nnz(C) and the status word back (one small copy + stream sync)
+// Numeric pass (ws_spgemm_numeric): one launch per non-empty class, no sync.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+
+#include "ws_internal.cuh"
+#include "ws_spgemm.h"
+
+using namespace wsk;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+// Process-wide tuning (ws_set_tuning).
+int64_t g_hash_max = kMaxHashProducts;
+int g_run_limit = 64;
+int g_dense_width = 0;  // 0 = default per value type
+constexpr int kLongRowThreshold = 128;
+
+ws_status_t fail(ws_status_t st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+ws_status_t fail(ws_status_t st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+ws_status_t cuda_fail(cudaError_t e, const char* what) {
+  return fail(WS_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define WS_CUDA(call, what)                     \
+  do {                                          \
+    cudaError_t e_ = (call);                    \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Grow-only stream-ordered device buffer.
+struct DevBuf {
+  void* ptr = nullptr;
+  size_t bytes = 0;
+  ws_status_t reserve(size_t need, cudaStream_t s) {
+    if (need <= bytes) return WS_OK;
+    if (ptr) {
+      cudaError_t e = cudaFreeAsync(ptr, s);
+      ptr = nullptr;
+      bytes = 0;
+      if (e != cudaSuccess) return cuda_fail(e, "cudaFreeAsync");
+    }
+    size_t want = need + need / 8;
+    cudaError_t e = cudaMallocAsync(&ptr, want, s);
+    if (e != cudaSuccess) {
+      ptr = nullptr;
+      return fail(WS_ERR_ALLOC, "cudaMallocAsync(%zu bytes): %s", want, cudaGetErrorString(e));
+    }
+    bytes = want;
+    return WS_OK;
+  }
+  void release() {
+    if (ptr) cudaFree(ptr);
+    ptr = nullptr;
+    bytes = 0;
+  }
+};
+
+struct Plan {
+  DevBuf rows;    // per-row arrays + summary + scan partials
+  DevBuf slices;  // dense-window slice arrays
+  DevSummary* host_sum = nullptr;  // pinned
+  // carved pointers
+  DevSummary* dsum = nullptr;
+  int32_t* perm = nullptr;
+  uint8_t* cls = nullptr;
+  int32_t* lo = nullptr;
+  int32_t* hi = nullptr;
+  int32_t* long_rows = nullptr;
+  int32_t* sort_list = nullptr;
+  int64_t* partials = nullptr;
+  int32_t* slice_row = nullptr;
+  int32_t* slice_idx = nullptr;
+  int32_t* slice_first = nullptr;
+  int32_t* slice_cnt = nullptr;
+  // results of the last symbolic pass
+  bool ready = false;
+  const void* A = nullptr;
+  const void* B = nullptr;
+  int64_t a_nnz = -1, b_nnz = -1;
+  int64_t seg_count[kNumSegs] = {};
+  int64_t seg_offset[kNumSegs + 1] = {};
+  int64_t n_sort = 0, n_empty = 0, dense_slices = 0, products = 0;
+  int log2_group = 5;
+  int dense_width = 0;
+  int run_limit = 64;
+  int sym_launches = 0, num_launches = 0;
+};
+
+}  // namespace
+
+struct ws_csr_s {
+  int64_t nrows = 0, ncols = 0, nnz = 0;
+  int64_t* rowptr = nullptr;
+  int32_t* colidx = nullptr;
+  void* vals = nullptr;
+  ws_dtype_t dtype = WS_F64;
+  int device = 0;
+  Plan* plan = nullptr;
+};
+
+namespace {
+
+int num_sms_of(int device) {
+  static int cached_dev = -1, cached = 0;
+  if (cached_dev != device) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device) != cudaSuccess || n <= 0) n = 1;
+    cached = n;
+    cached_dev = device;
+  }
+  return cached;
+}
+
+int log2_group_for(const ws_csr_s* B) {
+  const double avg = B->nrows > 0 ? static_cast<double>(B->nnz) / static_cast<double>(B->nrows) : 0.0;
+  if (avg <= 4.0) return 2;
+  if (avg <= 8.0) return 3;
+  if (avg <= 16.0) return 4;
+  return 5;
+}
+
+ws_status_t read_summary(Plan* pl, cudaStream_t s) {
+  WS_CUDA(cudaMemcpyAsync(pl->host_sum, pl->dsum, sizeof(DevSummary), cudaMemcpyDeviceToHost, s),
+          "cudaMemcpyAsync(summary)");
+  WS_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+  return WS_OK;
+}
+
+ws_status_t device_status(const DevSummary& hs) {
+  if (hs.status == 0) return WS_OK;
+  return fail(WS_ERR_DEVICE, "device status 0x%x (probe=%d rank=%d count=%d sortcap=%d)", hs.status,
+              !!(hs.status & kErrProbe), !!(hs.status & kErrRank), !!(hs.status & kErrCount),
+              !!(hs.status & kErrSortCap));
+}
+
+template <typename T>
+RowPlan<T> make_rowplan(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl) {
+  RowPlan<T> p{};
+  p.A = {A->rowptr, A->colidx, static_cast<const T*>(A->vals)};
+  p.B = {B->rowptr, B->colidx, static_cast<const T*>(B->vals)};
+  p.c_rowptr = C->rowptr;
+  p.c_colidx = C->colidx;
+  p.c_vals = static_cast<T*>(C->vals);
+  p.perm = pl->perm;
+  p.cls = pl->cls;
+  p.lo = pl->lo;
+  p.hi = pl->hi;
+  p.sort_list = pl->sort_list;
+  p.slice_row = pl->slice_row;
+  p.slice_idx = pl->slice_idx;
+  p.slice_first = pl->slice_first;
+  p.slice_cnt = pl->slice_cnt;
+  p.sum = pl->dsum;
+  p.log2_group = pl->log2_group;
+  p.run_limit = pl->run_limit;
+  p.dense_width = pl->dense_width;
+  return p;
+}
+
+ws_status_t carve_rows(Plan* pl, int64_t m, cudaStream_t s) {
+  const int64_t nb = scan_partials_needed(m);
+  size_t off = 0;
+  const size_t o_sum = off; off = align_up(off + sizeof(DevSummary), 256);
+  const size_t o_perm = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_lo = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_hi = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_long = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_sort = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
+  const size_t o_cls = off; off = align_up(off + static_cast<size_t>(m), 256);
+  ws_status_t st = pl->rows.reserve(off, s);
+  if (st != WS_OK) return st;
+  char* b = static_cast<char*>(pl->rows.ptr);
+  pl->dsum = reinterpret_cast<DevSummary*>(b + o_sum);
+  pl->perm = reinterpret_cast<int32_t*>(b + o_perm);
+  pl->lo = reinterpret_cast<int32_t*>(b + o_lo);
+  pl->hi = reinterpret_cast<int32_t*>(b + o_hi);
+  pl->long_rows = reinterpret_cast<int32_t*>(b + o_long);
+  pl->sort_list = reinterpret_cast<int32_t*>(b + o_sort);
+  pl->partials = reinterpret_cast<int64_t*>(b + o_part);
+  pl->cls = reinterpret_cast<uint8_t*>(b + o_cls);
+  return WS_OK;
+}
+
+ws_status_t carve_slices(Plan* pl, int64_t nslices, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(nslices > 0 ? nslices : 1);
+  const size_t each = align_up(4 * n, 256);
+  ws_status_t st = pl->slices.reserve(4 * each, s);
+  if (st != WS_OK) return st;
+  char* b = static_cast<char*>(pl->slices.ptr);
+  pl->slice_row = reinterpret_cast<int32_t*>(b);
+  pl->slice_idx = reinterpret_cast<int32_t*>(b + each);
+  pl->slice_first = reinterpret_cast<int32_t*>(b + 2 * each);
+  pl->slice_cnt = reinterpret_cast<int32_t*>(b + 3 * each);
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, cudaStream_t s,
+                          int64_t* nnz_out) {
+  const int64_t m = A->nrows;
+  const int dev = C->device;
+  const int sms = num_sms_of(dev);
+  pl->ready = false;
+  pl->sym_launches = 0;
+  pl->log2_group = log2_group_for(B);
+  pl->run_limit = g_run_limit;
+  pl->dense_width = g_dense_width > 0 ? g_dense_width : (sizeof(T) == 8 ? 8192 : 16384);
+
+  ws_status_t st = carve_rows(pl, m, s);
+  if (st != WS_OK) return st;
+  WS_CUDA(cudaMemsetAsync(pl->dsum, 0, sizeof(DevSummary), s), "cudaMemsetAsync(summary)");
+  WS_CUDA(cudaMemsetAsync(C->rowptr, 0, sizeof(int64_t), s), "cudaMemsetAsync(rowptr[0])");
+
+  RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
+  if (m > 0) {
+    AnalyzeParams ap{m, g_hash_max, pl->dense_width, kLongRowThreshold};
+    launch_analyze<T>(p, ap, pl->long_rows, sms, s, &pl->sym_launches);
+    WS_CUDA(cudaGetLastError(), "analyze launch");
+  }
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  const DevSummary& hs = *pl->host_sum;
+  int64_t off = 0;
+  for (int g = 0; g < kNumSegs; ++g) {
+    pl->seg_count[g] = hs.seg_count[g];
+    pl->seg_offset[g] = off;
+    off += hs.seg_count[g];
+  }
+  pl->seg_offset[kNumSegs] = off;
+  pl->n_empty = hs.n_empty;
+  pl->products = hs.products;
+  pl->dense_slices = hs.dense_slices;
+  if (pl->dense_slices > INT32_MAX) return fail(WS_ERR_OVERFLOW, "too many dense-window slices (%lld)", (long long)pl->dense_slices);
+
+  if (off > 0) {
+    launch_scatter<T>(p, m, pl->seg_offset, sms, s, &pl->sym_launches);
+  }
+  if (pl->seg_count[kSegDense] > 0) {
+    st = carve_slices(pl, pl->dense_slices, s);
+    if (st != WS_OK) return st;
+    p = make_rowplan<T>(A, B, C, pl);
+    p.seg_begin = pl->seg_offset[kSegDense];
+    p.seg_len = pl->seg_count[kSegDense];
+    launch_dense_slices<T>(p, pl->slice_row, pl->slice_idx, pl->slice_first, sms, s, &pl->sym_launches);
+    launch_dense<T>(p, pl->dense_slices, false, sms, s, &pl->sym_launches);
+  }
+  for (int b = 0; b < kNumHashBins; ++b) {
+    const int g = kSegHash0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_hash<T>(p, b, false, sms, s, &pl->sym_launches);
+  }
+  launch_scan(C->rowptr, m, pl->partials, pl->dsum, s, &pl->sym_launches);
+  WS_CUDA(cudaGetLastError(), "symbolic launches");
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  st = device_status(*pl->host_sum);
+  if (st != WS_OK) return st;
+  pl->n_sort = pl->host_sum->n_sort;
+  C->nnz = m > 0 ? pl->host_sum->nnz : 0;
+  pl->A = A;
+  pl->B = B;
+  pl->a_nnz = A->nnz;
+  pl->b_nnz = B->nnz;
+  pl->ready = true;
+  *nnz_out = C->nnz;
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, cudaStream_t s) {
+  const int sms = num_sms_of(C->device);
+  pl->num_launches = 0;
+  RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
+  if (pl->seg_count[kSegDirect] > 0) {
+    p.seg_begin = pl->seg_offset[kSegDirect];
+    p.seg_len = pl->seg_count[kSegDirect];
+    launch_direct<T>(p, sms, s, &pl->num_launches);
+  }
+  for (int b = 0; b < kNumHashBins; ++b) {
+    const int g = kSegHash0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_hash<T>(p, b, true, sms, s, &pl->num_launches);
+  }
+  if (pl->n_sort > 0) launch_sort<T>(p, pl->n_sort, sms, s, &pl->num_launches);
+  if (pl->seg_count[kSegDense] > 0) {
+    p.seg_begin = pl->seg_offset[kSegDense];
+    p.seg_len = pl->seg_count[kSegDense];
+    launch_dense<T>(p, pl->dense_slices, true, sms, s, &pl->num_launches);
+  }
+  WS_CUDA(cudaGetLastError(), "numeric launches");
+  return WS_OK;
+}
+
+ws_status_t check_handle(const ws_csr_s* h, const char* name) {
+  if (!h) return fail(WS_ERR_INVALID_ARG, "%s is NULL", name);
+  return WS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ws_status_t ws_csr_create(ws_csr_t* out, int64_t nrows, int64_t ncols, int64_t nnz, int64_t* rowptr,
+                          int32_t* colidx, void* vals, ws_dtype_t dtype, int validate, ws_stream_t stream) {
+  g_last_error.clear();
+  if (!out) return fail(WS_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (nrows < 0 || ncols < 0 || nnz < 0) return fail(WS_ERR_INVALID_ARG, "negative size");
+  if (nrows > INT32_MAX - 1 || ncols > INT32_MAX)
+    return fail(WS_ERR_OVERFLOW, "nrows/ncols exceed the int32 index range");
+  if (dtype != WS_F32 && dtype != WS_F64) return fail(WS_ERR_INVALID_ARG, "unknown dtype %d", (int)dtype);
+  if (!rowptr) return fail(WS_ERR_INVALID_ARG, "rowptr is NULL");
+  if (nnz > 0 && (!colidx || !vals)) return fail(WS_ERR_INVALID_ARG, "colidx/vals NULL with nnz > 0");
+  int dev = 0;
+  WS_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  if (validate) {
+    DevSummary* d = nullptr;
+    DevSummary h{};
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    WS_CUDA(cudaMallocAsync(reinterpret_cast<void**>(&d), sizeof(DevSummary), s), "cudaMallocAsync(validate)");
+    h.bad_row = INT32_MAX;
+    cudaError_t e = cudaMemcpyAsync(d, &h, sizeof(h), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && nrows > 0) {
+      launch_validate(rowptr, colidx, nrows, ncols, nnz, d, num_sms_of(dev), s);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&h, d, sizeof(h), cudaMemcpyDeviceToHost, s);
+    cudaFreeAsync(d, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "validation");
+    if (nrows == 0) {
+      int64_t r0 = -1;
+      WS_CUDA(cudaMemcpy(&r0, rowptr, sizeof(r0), cudaMemcpyDeviceToHost), "cudaMemcpy(rowptr[0])");
+      if (r0 != 0 || nnz != 0) return fail(WS_ERR_INVALID_CSR, "empty matrix needs rowptr[0] = 0 and nnz = 0");
+    }
+    if (h.status & kErrInvalidCsr)
+      return fail(WS_ERR_INVALID_CSR, "CSR invariants violated (first bad row %d)", h.bad_row);
+  }
+  ws_csr_s* hnd = new (std::nothrow) ws_csr_s;
+  if (!hnd) return fail(WS_ERR_ALLOC, "host allocation failed");
+  hnd->nrows = nrows;
+  hnd->ncols = ncols;
+  hnd->nnz = nnz;
+  hnd->rowptr = rowptr;
+  hnd->colidx = colidx;
+  hnd->vals = vals;
+  hnd->dtype = dtype;
+  hnd->device = dev;
+  *out = hnd;
+  return WS_OK;
+}
+
+ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_out, ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  if (!nnz_out) return fail(WS_ERR_INVALID_ARG, "nnz_out is NULL");
+  if (C == A || C == B) return fail(WS_ERR_INVALID_ARG, "C must be a separate output handle");
+  if (A->ncols != B->nrows)
+    return fail(WS_ERR_SHAPE, "A is %lldx%lld but B is %lldx%lld", (long long)A->nrows, (long long)A->ncols,
+                (long long)B->nrows, (long long)B->ncols);
+  if (C->nrows != A->nrows || C->ncols != B->ncols)
+    return fail(WS_ERR_SHAPE, "C is %lldx%lld, expected %lldx%lld", (long long)C->nrows, (long long)C->ncols,
+                (long long)A->nrows, (long long)B->ncols);
+  if (A->dtype != B->dtype || C->dtype != A->dtype) return fail(WS_ERR_DTYPE, "A, B and C dtypes differ");
+  if (A->nnz > 0 && B->nrows == 0) return fail(WS_ERR_INVALID_CSR, "A has entries but B has no rows");
+  if (!C->plan) {
+    C->plan = new (std::nothrow) Plan;
+    if (!C->plan) return fail(WS_ERR_ALLOC, "host allocation failed");
+  }
+  Plan* pl = C->plan;
+  if (!pl->host_sum) {
+    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&pl->host_sum), sizeof(DevSummary));
+    if (e != cudaSuccess) {
+      pl->host_sum = nullptr;
+      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
+    }
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  C->nnz = -1;
+  if (A->dtype == WS_F64) return symbolic_impl<double>(A, B, C, pl, s, nnz_out);
+  return symbolic_impl<float>(A, B, C, pl, s, nnz_out);
+}
+
+ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                              ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  Plan* pl = C->plan;
+  if (!pl || !pl->ready) return fail(WS_ERR_STATE, "numeric called before a successful symbolic pass");
+  if (pl->A != A || pl->B != B || pl->a_nnz != A->nnz || pl->b_nnz != B->nnz)
+    return fail(WS_ERR_STATE, "numeric called with other operands than the symbolic pass");
+  if (C->nnz > 0 && (!c_colidx || !c_vals)) return fail(WS_ERR_INVALID_ARG, "c_colidx/c_vals NULL with nnz(C) > 0");
+  C->colidx = c_colidx;
+  C->vals = c_vals;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (A->dtype == WS_F64) return numeric_impl<double>(A, B, C, pl, s);
+  return numeric_impl<float>(A, B, C, pl, s);
+}
+
+ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
+  g_last_error.clear();
+  if (!C) return fail(WS_ERR_INVALID_ARG, "C is NULL");
+  Plan* pl = C->plan;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (!pl || !pl->host_sum || !pl->dsum) {
+    WS_CUDA(cudaStreamSynchronize(s), "cudaStreamSynchronize");
+    return WS_OK;
+  }
+  ws_status_t st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  return device_status(*pl->host_sum);
+}
+
+ws_status_t ws_csr_destroy(ws_csr_t h) {
+  if (!h) return WS_OK;
+  if (h->plan) {
+    if (h->plan->rows.ptr || h->plan->slices.ptr) cudaDeviceSynchronize();
+    h->plan->rows.release();
+    h->plan->slices.release();
+    if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
+    delete h->plan;
+  }
+  delete h;
+  return WS_OK;
+}
+
+const char* ws_status_string(ws_status_t st) {
+  switch (st) {
+    case WS_OK: return "ok";
+    case WS_ERR_INVALID_ARG: return "invalid argument";
+    case WS_ERR_INVALID_CSR: return "invalid CSR matrix";
+    case WS_ERR_SHAPE: return "shape mismatch";
+    case WS_ERR_DTYPE: return "dtype mismatch";
+    case WS_ERR_OVERFLOW: return "size overflow";
+    case WS_ERR_ALLOC: return "allocation failed";
+    case WS_ERR_CUDA: return "CUDA error";
+    case WS_ERR_DEVICE: return "device-side failure";
+    case WS_ERR_STATE: return "calls out of order";
+  }
+  return "unknown status";
+}
+
+const char* ws_last_error(void) { return g_last_error.c_str(); }
+
+ws_status_t ws_csr_nnz(ws_csr_t h, int64_t* nnz_out) {
+  if (!h || !nnz_out) return fail(WS_ERR_INVALID_ARG, "NULL argument");
+  *nnz_out = h->nnz;
+  return WS_OK;
+}
+
+ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
+  if (!C || !info || n < 0) return fail(WS_ERR_INVALID_ARG, "NULL argument");
+  const Plan* pl = C->plan;
+  int64_t v[9] = {0, 0, 0, 0, 0, 0, 0, 0, 0};
+  if (pl) {
+    int64_t hash_rows = 0;
+    for (int b = 0; b < kNumHashBins; ++b) hash_rows += pl->seg_count[kSegHash0 + b];
+    v[0] = pl->n_empty;
+    v[1] = pl->seg_count[kSegDirect];
+    v[2] = hash_rows;
+    v[3] = pl->n_sort;
+    v[4] = pl->seg_count[kSegDense];
+    v[5] = pl->dense_slices;
+    v[6] = pl->products;
+    v[7] = pl->sym_launches;
+    v[8] = pl->num_launches;
+  }
+  for (int i = 0; i < n && i < 9; ++i) info[i] = v[i];
+  return WS_OK;
+}
+
+ws_status_t ws_set_tuning(int key, int64_t value) {
+  switch (key) {
+    case 1:
+      if (value < 0 || value > kMaxHashProducts) return fail(WS_ERR_INVALID_ARG, "hash limit out of range");
+      g_hash_max = value;
+      return WS_OK;
+    case 2:
+      if (value < 1 || value > 4096) return fail(WS_ERR_INVALID_ARG, "run limit out of range");
+      g_run_limit = static_cast<int>(value);
+      return WS_OK;
+    case 3:
+      if (value != 0 && (value < 1024 || value > 16384 || value % 1024 != 0))
+        return fail(WS_ERR_INVALID_ARG, "dense width must be 0 or a multiple of 1024 in [1024, 16384]");
+      g_dense_width = static_cast<int>(value);
+      return WS_OK;
+  }
+  return fail(WS_ERR_INVALID_ARG, "unknown tuning key %d", key);
+}
+
+}  // extern "C"

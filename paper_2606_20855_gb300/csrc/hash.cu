@@ -1,0 +1,313 @@
+// Hash-bin rows: per-row shared-memory hash workspace with a monotone hash and
+// sort-free ranking.
+//
+// Workspace.  Row i of C = A*B is the sum of the scaled rows A[i,k] * B[k,:]
+// (Gustavson's algorithm, Sec. 5.1).  One thread team (one or more warps)
+// owns the row, so the team's table is the private workspace w of the paper
+// and the row's output segment is written by nobody else.  Inside the team,
+// concurrent updates of one workspace entry use shared-memory atomics (the
+// atomic-level protection of Sec. 4).
+//
+// Monotone hash.  Every product column of the row lies in [lo, hi] (B's rows
+// are sorted).  The home slot of column c is
+//     h(c) = floor((c - lo) * T / span),  span = hi - lo + 1,
+// (h(c) = c - lo when span <= T), which never decreases as c grows.  With
+// linear probing and no wrap-around, every key's home lies inside the run of
+// occupied slots ("cluster") that holds the key, so keys of an earlier
+// cluster are smaller than keys of a later one.  Hence the sorted position of
+// the key in slot s is
+//     (#occupied slots before s) - (s - cluster_start) + #{keys of s's cluster < key(s)}
+// and the row is written in sorted column order without a sort.  The
+// symbolic pass checks each row's table for a wrap-around or a cluster longer
+// than the ranking limit and re-routes such rows to the sorting path.  The
+// set of occupied slots of a linear-probing table does not depend on the
+// insertion order, so the numeric pass (same keys, same table, same hash)
+// sees exactly the clusters the symbolic pass checked.
+//
+// Table sizes: bin b holds rows with at most 32 << b products in 64 << b
+// slots, so the load factor is at most 1/2.
+#include "ws_internal.cuh"
+
+namespace wsk {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kEmptyKey = -1;
+
+template <int WPR>
+__device__ __forceinline__ void team_sync() {
+  if constexpr (WPR == 1) {
+    __syncwarp();
+  } else {
+    __syncthreads();
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ void atomic_add_value(T* addr, T v) {
+  atomicAdd(addr, v);
+}
+
+// Inserts key c (and adds v when NUMERIC) into the table; returns 1 if the
+// key was new, 0 if it was present, -1 if the whole table was probed.
+template <bool NUMERIC, typename T>
+__device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint32_t mask, int c, T v,
+                                            bool& wrapped) {
+  volatile int* vk = keys;
+  for (uint32_t n = 0; n <= mask; ++n) {
+    int cur = vk[h];
+    if (cur == kEmptyKey) {
+      cur = atomicCAS(&keys[h], kEmptyKey, c);
+      if (cur == kEmptyKey) {
+        if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
+        return 1;
+      }
+    }
+    if (cur == c) {
+      if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
+      return 0;
+    }
+    h = (h + 1) & mask;
+    wrapped |= (h == 0);
+  }
+  return -1;
+}
+
+// True if the table holds a run of more than `limit` occupied slots.  Called
+// by one full warp; every lane returns the same value.
+__device__ __forceinline__ bool has_long_run(const int* keys, int nslots, int limit, int lane) {
+  int carry = 0;
+  bool bad = false;
+  for (int base = 0; base < nslots; base += 32) {
+    const unsigned m = __ballot_sync(kFull, keys[base + lane] != kEmptyKey);
+    if (m == kFull) {
+      carry += 32;
+      bad |= carry > limit;
+    } else {
+      bad |= carry + (__ffs(~m) - 1) > limit;
+      if (limit < 31) {
+        unsigned x = m;
+        for (int j = 0; j < limit; ++j) x &= x >> 1;
+        bad |= x != 0;
+      }
+      carry = __clz(~m);
+    }
+  }
+  return bad;
+}
+
+template <typename T>
+__device__ __forceinline__ void clear_values(T* vals, int n, int t, int nt) {
+  int4* v4 = reinterpret_cast<int4*>(vals);
+  const int n4 = static_cast<int>(n * sizeof(T) / sizeof(int4));
+  for (int s = t; s < n4; s += nt) v4[s] = make_int4(0, 0, 0, 0);
+}
+
+// LOGT: log2 of table slots; WPR: warps per row team; RPC: row teams per CTA.
+template <typename T, int LOGT, int WPR, int RPC, bool NUMERIC>
+__global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan<T> p, const uint8_t my_cls) {
+  static_assert(WPR == 1 || RPC == 1, "multi-warp row teams use the whole CTA");
+  constexpr int kT = 1 << LOGT;
+  constexpr uint32_t kMask = kT - 1;
+  constexpr int kNT = 32 * WPR;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ int s_warp[WPR > 1 ? WPR : 1];
+  __shared__ int s_flags;
+
+  const int sub = threadIdx.x / kNT;
+  const int t = threadIdx.x % kNT;
+  const int lane = threadIdx.x & 31;
+  const int warp = t >> 5;
+  int* keys = reinterpret_cast<int*>(smem_raw) + sub * kT;
+  T* vals = nullptr;
+  if constexpr (NUMERIC) vals = reinterpret_cast<T*>(reinterpret_cast<int*>(smem_raw) + RPC * kT) + sub * kT;
+
+  const int lg = p.log2_group;
+  const int gsize = 1 << lg;
+  const int grp = t >> lg;
+  const int gl = t & (gsize - 1);
+  const int ngrp = kNT >> lg;
+
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * RPC + sub; r < p.seg_len;
+       r += static_cast<int64_t>(gridDim.x) * RPC) {
+    const int32_t row = p.perm[p.seg_begin + r];
+    if constexpr (NUMERIC) {
+      if (p.cls[row] != my_cls) continue;  // re-routed to the sorting path (uniform over the team)
+    }
+    const int lo = p.lo[row];
+    const uint32_t span = static_cast<uint32_t>(p.hi[row] - lo) + 1u;
+    const bool ident = span <= static_cast<uint32_t>(kT);
+    const unsigned long long mul = ident ? 0ull : ((static_cast<unsigned long long>(kT) << 32) / span);
+
+    // Clear the workspace (w .= 0).
+    {
+      int4* k4 = reinterpret_cast<int4*>(keys);
+      for (int s = t; s < kT / 4; s += kNT) k4[s] = make_int4(kEmptyKey, kEmptyKey, kEmptyKey, kEmptyKey);
+      if constexpr (NUMERIC) clear_values(vals, kT, t, kNT);
+      if constexpr (WPR > 1) {
+        if (t < WPR) s_warp[t] = 0;
+        if (t == 0) s_flags = 0;
+      }
+    }
+    team_sync<WPR>();
+
+    // Accumulate: w[j] += A[i,k] * B[k,j] for every stored A[i,k], B[k,j].
+    int my_new = 0;
+    bool wrapped = false, failed = false;
+    const int64_t pa_end = p.A.rowptr[row + 1];
+    for (int64_t pa = p.A.rowptr[row] + grp; pa < pa_end; pa += ngrp) {
+      const int k = p.A.colidx[pa];
+      T av = T(0);
+      if constexpr (NUMERIC) av = p.A.vals[pa];
+      const int64_t qe = p.B.rowptr[k + 1];
+      for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
+        const int c = p.B.colidx[q];
+        T v = T(0);
+        if constexpr (NUMERIC) v = av * p.B.vals[q];
+        const uint32_t d = static_cast<uint32_t>(c - lo);
+        const uint32_t h = ident ? d : static_cast<uint32_t>((static_cast<unsigned long long>(d) * mul) >> 32);
+        const int res = probe_insert<NUMERIC>(keys, vals, h, kMask, c, v, wrapped);
+        my_new += res > 0;
+        failed |= res < 0;
+      }
+    }
+
+    if constexpr (!NUMERIC) {
+      // Count the distinct columns, check the table for the ranking condition.
+      int cnt = my_new;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+      const int flags = (__any_sync(kFull, wrapped) ? 1 : 0) | (__any_sync(kFull, failed) ? 2 : 0);
+      if constexpr (WPR > 1) {
+        if (lane == 0) {
+          atomicAdd(&s_warp[0], cnt);
+          atomicOr(&s_flags, flags);
+        }
+      }
+      team_sync<WPR>();
+      if (warp == 0) {
+        int total = cnt, fl = flags;
+        if constexpr (WPR > 1) {
+          total = s_warp[0];
+          fl = s_flags;
+        }
+        const bool long_run = has_long_run(keys, kT, p.run_limit, lane);
+        if (lane == 0) {
+          p.c_rowptr[row + 1] = total;
+          if (fl & 2) atomicOr(&p.sum->status, kErrProbe);
+          if ((fl & 1) || long_run) {
+            p.cls[row] = kClsSort;
+            p.sort_list[atomicAdd(&p.sum->n_sort, 1)] = row;
+          }
+        }
+      }
+      team_sync<WPR>();
+    } else {
+      team_sync<WPR>();
+      // Rank and write: each warp ranks a contiguous range of slots.
+      constexpr int kPerWarp = kT / WPR;
+      const int s_begin = warp * kPerWarp;
+      int carry = 0;
+      if constexpr (WPR > 1) {
+        int occ = 0;
+        for (int s = s_begin + lane; s < s_begin + kPerWarp; s += 32) occ += keys[s] != kEmptyKey;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) occ += __shfl_xor_sync(kFull, occ, o);
+        if (lane == 0) s_warp[warp] = occ;
+        team_sync<WPR>();
+        for (int w = 0; w < warp; ++w) carry += s_warp[w];
+      }
+      const int64_t base = p.c_rowptr[row];
+      const int64_t cnt = p.c_rowptr[row + 1] - base;
+      const int limit = p.run_limit;
+      bool rank_err = false, count_err = false;
+      for (int c0 = s_begin; c0 < s_begin + kPerWarp; c0 += 32) {
+        const int s = c0 + lane;
+        const int key = keys[s];
+        const bool occ = key != kEmptyKey;
+        const unsigned m = __ballot_sync(kFull, occ);
+        if (occ) {
+          const int before = carry + __popc(m & ((1u << lane) - 1u));
+          int rk = 0;
+          int cs = s;
+          int steps = 0;
+          while (cs > 0 && steps < limit) {
+            const int kk = keys[cs - 1];
+            if (kk == kEmptyKey) break;
+            rk += kk < key;
+            --cs;
+            ++steps;
+          }
+          if (cs > 0 && steps == limit && keys[cs - 1] != kEmptyKey) rank_err = true;
+          int u = s + 1;
+          for (steps = 0; u < kT && steps < limit; ++u, ++steps) {
+            const int kk = keys[u];
+            if (kk == kEmptyKey) break;
+            rk += kk < key;
+          }
+          if (u < kT && steps == limit && keys[u] != kEmptyKey) rank_err = true;
+          const int64_t pos = static_cast<int64_t>(before) - (s - cs) + rk;
+          if (pos >= 0 && pos < cnt) {
+            p.c_colidx[base + pos] = key;
+            p.c_vals[base + pos] = vals[s];
+          } else {
+            count_err = true;
+          }
+        }
+        carry += __popc(m);
+      }
+      if (WPR == 1 || warp == WPR - 1) {
+        if (carry != cnt) count_err = true;
+      }
+      if (__any_sync(kFull, rank_err) && lane == 0) atomicOr(&p.sum->status, kErrRank);
+      if (__any_sync(kFull, count_err) && lane == 0) atomicOr(&p.sum->status, kErrCount);
+      if (__any_sync(kFull, failed) && lane == 0) atomicOr(&p.sum->status, kErrProbe);
+      team_sync<WPR>();
+    }
+  }
+}
+
+template <typename T, int LOGT, int WPR, int RPC>
+void launch_bin(const RowPlan<T>& p, bool numeric, int bin, int num_sms, cudaStream_t s) {
+  constexpr int kT = 1 << LOGT;
+  const size_t smem = static_cast<size_t>(RPC) * kT * (sizeof(int) + (numeric ? sizeof(T) : 0));
+  const int threads = 32 * WPR * RPC;
+  auto kern = numeric ? hash_rows_kernel<T, LOGT, WPR, RPC, true> : hash_rows_kernel<T, LOGT, WPR, RPC, false>;
+  static bool configured[2] = {false, false};
+  if (!configured[numeric]) {
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    configured[numeric] = true;
+  }
+  int per_sm = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (p.seg_len + RPC - 1) / RPC;
+  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  kern<<<static_cast<int>(grid), threads, smem, s>>>(p, static_cast<uint8_t>(kClsHash0 + bin));
+}
+
+}  // namespace
+
+template <typename T>
+void launch_hash(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches) {
+  switch (bin) {
+    case 0: launch_bin<T, 6, 1, 8>(p, numeric, bin, num_sms, s); break;
+    case 1: launch_bin<T, 7, 1, 8>(p, numeric, bin, num_sms, s); break;
+    case 2: launch_bin<T, 8, 1, 8>(p, numeric, bin, num_sms, s); break;
+    case 3: launch_bin<T, 9, 1, 8>(p, numeric, bin, num_sms, s); break;
+    case 4: launch_bin<T, 10, 1, 4>(p, numeric, bin, num_sms, s); break;
+    case 5: launch_bin<T, 11, 2, 1>(p, numeric, bin, num_sms, s); break;
+    case 6: launch_bin<T, 12, 4, 1>(p, numeric, bin, num_sms, s); break;
+    case 7: launch_bin<T, 13, 8, 1>(p, numeric, bin, num_sms, s); break;
+    default: return;
+  }
+  *launches += 1;
+}
+
+template void launch_hash<float>(const RowPlan<float>&, int, bool, int, cudaStream_t, int*);
+template void launch_hash<double>(const RowPlan<double>&, int, bool, int, cudaStream_t, int*);
+
+}  // namespace wsk

@@ -1,0 +1,169 @@
+// Internal declarations shared by the CUDA translation units of the SpGEMM library.
+//
+// Row classes.  The symbolic pass sorts every output row i of C = A*B into one
+// class by its product count ub_i = sum over stored A[i,k] of |B[k,:]| (the
+// work of the row, which is data dependent and unknown before the pass --
+// the load-balance problem of Sec. 1):
+//   empty         ub_i = 0                       -> no output
+//   direct        exactly one stored A[i,k]      -> C[i,:] = A[i,k] * B[k,:]
+//   hash bin b    ub_i <= 32 << b (b = 0..7)     -> shared-memory hash workspace of
+//                                                  64 << b slots, sort-free ranking
+//   sort          a hash row whose table showed a long run of occupied slots
+//                 (or wrapped) -> shared-memory hash + bitonic sort
+//   dense window  ub_i above the hash limit      -> column slices of the row, each a
+//                                                  dense bitmap + value workspace
+// Each class is a different realisation of the per-row workspace w of
+// Gustavson's algorithm (Sec. 5.1); every row is written by exactly one
+// thread team (or, for dense-window rows, each column slice by one team),
+// so C's segments are disjoint (the shard pattern, Sec. 4).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace wsk {
+
+constexpr int kNumHashBins = 8;
+constexpr int kMinHashLog = 6;  // bin b uses a table of 1 << (kMinHashLog + b) slots
+constexpr int kMaxHashProducts = 32 << (kNumHashBins - 1);  // 4096
+
+// Row class codes stored per row (uint8).
+constexpr uint8_t kClsEmpty = 0;
+constexpr uint8_t kClsDirect = 1;
+constexpr uint8_t kClsHash0 = 2;  // 2 .. 2 + kNumHashBins - 1
+constexpr uint8_t kClsDense = kClsHash0 + kNumHashBins;
+constexpr uint8_t kClsSort = kClsDense + 1;
+
+// Segments of the row permutation: direct rows, hash bins, dense-window rows.
+constexpr int kSegDirect = 0;
+constexpr int kSegHash0 = 1;
+constexpr int kSegDense = kSegHash0 + kNumHashBins;
+constexpr int kNumSegs = kSegDense + 1;
+
+// Device error flags (OR-ed into DevSummary::status).
+enum DevError : int {
+  kErrProbe = 1,       // a hash insert ran through a whole table (cannot happen at load <= 1/2)
+  kErrRank = 2,        // a run of occupied slots longer than the ranking limit in the numeric pass
+  kErrCount = 4,       // the numeric pass found a different entry count than the symbolic pass
+  kErrInvalidCsr = 8,  // validation found broken CSR invariants
+  kErrSortCap = 16,    // a sort-path row exceeded its workspace
+};
+
+// Counters shared between the kernels of one product and read back by the host.
+struct DevSummary {
+  long long nnz;       // nnz(C), written by the scan
+  long long products;  // sum of ub_i
+  long long dense_slices;
+  long long slice_cursor;
+  int status;
+  int n_sort;
+  int n_long;
+  int n_empty;
+  int bad_row;
+  int pad0;
+  int seg_count[kNumSegs];
+  int seg_cursor[kNumSegs];
+};
+
+// Read-only view of an input CSR matrix.
+template <typename T>
+struct CsrView {
+  const int64_t* rowptr;
+  const int32_t* colidx;
+  const T* vals;
+};
+
+// Everything the row kernels need about one product.
+template <typename T>
+struct RowPlan {
+  CsrView<T> A;
+  CsrView<T> B;
+  int64_t* c_rowptr;   // C.rowptr; symbolic writes counts to [i + 1] then scans in place
+  int32_t* c_colidx;   // numeric only
+  T* c_vals;           // numeric only
+  int32_t* perm;       // rows grouped by segment
+  uint8_t* cls;        // row class per row
+  int32_t* lo;         // smallest column any product of the row can hit
+  int32_t* hi;         // largest such column
+  int32_t* sort_list;  // rows rerouted to the sorting path
+  const int32_t* slice_row;    // dense-window slices: row, slice index, first slice of the row
+  const int32_t* slice_idx;
+  const int32_t* slice_first;
+  int32_t* slice_cnt;          // entries per dense-window slice
+  DevSummary* sum;
+  int64_t seg_begin;   // first position in perm of the segment a kernel processes
+  int64_t seg_len;     // rows in that segment
+  int log2_group;      // lanes per stored A entry when walking B rows (1 << log2_group)
+  int run_limit;       // longest occupied run the sort-free ranking accepts
+  int dense_width;     // dense-window slice width in columns
+};
+
+// Host-side launchers (one translation unit each).
+struct AnalyzeParams {
+  int64_t m;
+  int64_t hash_max;  // largest ub that uses a hash bin
+  int dense_width;
+  int long_threshold;
+};
+template <typename T>
+void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, int num_sms,
+                    cudaStream_t s, int* launches);
+template <typename T>
+void launch_scatter(const RowPlan<T>& p, int64_t m, const int64_t* seg_offset, int num_sms, cudaStream_t s,
+                    int* launches);
+template <typename T>
+void launch_dense_slices(const RowPlan<T>& p, int32_t* slice_row, int32_t* slice_idx, int32_t* slice_first,
+                         int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_hash(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_dense(const RowPlan<T>& p, int64_t nslices, bool numeric, int num_sms, cudaStream_t s,
+                  int* launches);
+template <typename T>
+void launch_direct(const RowPlan<T>& p, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_sort(const RowPlan<T>& p, int64_t nrows, int num_sms, cudaStream_t s, int* launches);
+
+void launch_scan(int64_t* rowptr, int64_t m, int64_t* partials, DevSummary* sum, cudaStream_t s, int* launches);
+int64_t scan_partials_needed(int64_t m);
+
+void launch_validate(const int64_t* rowptr, const int32_t* colidx, int64_t nrows, int64_t ncols, int64_t nnz,
+                     DevSummary* sum, int num_sms, cudaStream_t s);
+
+// Dynamic shared memory needed by the dense-window kernel and the sort kernel.
+size_t dense_smem_bytes(int width, size_t value_bytes, bool numeric);
+size_t sort_smem_bytes(size_t value_bytes);
+constexpr int kSortTableLog = 13;  // sort path: 8192-slot table, up to 4096 entries
+
+// Exclusive prefix sum over the threads of a CTA of blockDim.x threads
+// (a multiple of 32, at most 1024).  `scratch` holds 32 values; returns this
+// thread's exclusive prefix and stores the CTA total in *total.  Every thread
+// of the CTA must call it.
+template <typename V>
+__device__ __forceinline__ V block_exclusive_scan(V x, V* scratch, V* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  V incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const V y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) scratch[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    V w = lane < nwarps ? scratch[lane] : V(0);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const V y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nwarps) scratch[lane] = w;  // inclusive scan of warp totals
+  }
+  __syncthreads();
+  const V warp_prefix = warp > 0 ? scratch[warp - 1] : V(0);
+  *total = scratch[nwarps - 1];
+  __syncthreads();
+  return warp_prefix + incl - x;
+}
+
+}  // namespace wsk

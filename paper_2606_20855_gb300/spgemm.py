@@ -1,0 +1,143 @@
+"""PyTorch-facing wrapper of the C ABI: CSR matrices in torch device memory.
+
+PyTorch provides device memory and the current stream; the product itself is
+computed entirely by libws_spgemm.so through the four ABI calls:
+
+    ws_csr_create(A), ws_csr_create(B), ws_csr_create(C)    -- borrow arrays
+    nnz = ws_spgemm_symbolic(A, B, C)   -- C.rowptr + nnz(C) (the declare step)
+    allocate C.colidx[nnz], C.vals[nnz] with torch
+    ws_spgemm_numeric(A, B, C, ...)     -- fill C (the update step)
+    ws_csr_destroy(...)
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+import torch
+
+from . import _abi
+
+
+_DTYPES = {torch.float32: _abi.WS_F32, torch.float64: _abi.WS_F64}
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+@dataclass
+class DeviceCSR:
+    """CSR matrix whose arrays live in torch CUDA tensors."""
+
+    nrows: int
+    ncols: int
+    rowptr: torch.Tensor  # int64 [nrows + 1]
+    colidx: torch.Tensor  # int32 [nnz]
+    vals: torch.Tensor  # float32 / float64 [nnz]
+
+    @property
+    def nnz(self) -> int:
+        return int(self.colidx.numel())
+
+    @property
+    def dtype(self) -> torch.dtype:
+        return self.vals.dtype
+
+    @classmethod
+    def from_host(cls, M, device="cuda", non_blocking: bool = False) -> "DeviceCSR":
+        """Copies a host CSR (numpy arrays rowptr/colidx/vals) to the device."""
+        def put(a, dt):
+            t = torch.from_numpy(np.ascontiguousarray(a)).to(dt)
+            return t.to(device, non_blocking=non_blocking)
+        return cls(int(M.nrows), int(M.ncols), put(M.rowptr, torch.int64), put(M.colidx, torch.int32),
+                   put(M.vals, torch.float32 if np.dtype(M.vals.dtype) == np.float32 else torch.float64))
+
+    def to_host(self):
+        return (self.rowptr.cpu().numpy(), self.colidx.cpu().numpy(), self.vals.cpu().numpy())
+
+    def _handle(self, validate: bool, stream: int) -> int:
+        if self.dtype not in _DTYPES:
+            raise TypeError(f"values must be float32 or float64, got {self.dtype}")
+        for t, dt in ((self.rowptr, torch.int64), (self.colidx, torch.int32)):
+            if t.dtype != dt or not t.is_cuda or not t.is_contiguous():
+                raise TypeError("rowptr/colidx must be contiguous CUDA int64/int32 tensors")
+        if self.rowptr.numel() != self.nrows + 1:
+            raise ValueError("rowptr must have nrows + 1 entries")
+        nnz = self.nnz
+        return _abi.ws_csr_create(self.nrows, self.ncols, nnz, self.rowptr.data_ptr(),
+                                  self.colidx.data_ptr() if nnz else 0, self.vals.data_ptr() if nnz else 0,
+                                  _DTYPES[self.dtype], validate, stream)
+
+
+class SpGEMM:
+    """A reusable product C = A*B: handles and the row plan persist across calls.
+
+    ``symbolic()`` returns nnz(C) (and synchronises the stream), ``numeric()``
+    queues the value pass and returns C as a :class:`DeviceCSR`.
+    """
+
+    def __init__(self, A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None):
+        if A.dtype != B.dtype:
+            raise TypeError("A and B must have the same value dtype")
+        self.A, self.B = A, B
+        s = _stream_handle(stream)
+        self._hA = self._hB = self._hC = None
+        self.device = A.rowptr.device
+        self._hA = A._handle(validate, s)
+        self._hB = B._handle(validate, s)
+        self.c_rowptr = torch.empty(A.nrows + 1, dtype=torch.int64, device=self.device)
+        self._hC = _abi.ws_csr_create(A.nrows, B.ncols, 0, self.c_rowptr.data_ptr(), 0, 0,
+                                      _DTYPES[A.dtype], False, s)
+        self.nnz = None
+
+    def symbolic(self, stream=None) -> int:
+        self.nnz = _abi.ws_spgemm_symbolic(self._hA, self._hB, self._hC, _stream_handle(stream))
+        return self.nnz
+
+    def numeric(self, out: DeviceCSR | None = None, stream=None) -> DeviceCSR:
+        if self.nnz is None:
+            raise RuntimeError("symbolic() must run before numeric()")
+        if out is None or out.nnz != self.nnz:
+            colidx = torch.empty(self.nnz, dtype=torch.int32, device=self.device)
+            vals = torch.empty(self.nnz, dtype=self.A.dtype, device=self.device)
+            out = DeviceCSR(self.A.nrows, self.B.ncols, self.c_rowptr, colidx, vals)
+        _abi.ws_spgemm_numeric(self._hA, self._hB, self._hC, out.colidx.data_ptr() if self.nnz else 0,
+                               out.vals.data_ptr() if self.nnz else 0, _stream_handle(stream))
+        return out
+
+    def wait(self, stream=None) -> None:
+        _abi.ws_spgemm_wait(self._hC, _stream_handle(stream))
+
+    def plan_info(self) -> dict:
+        return _abi.ws_spgemm_plan_info(self._hC)
+
+    def close(self) -> None:
+        for name in ("_hC", "_hB", "_hA"):
+            h = getattr(self, name, None)
+            if h:
+                _abi.ws_csr_destroy(h)
+                setattr(self, name, None)
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def spgemm(A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None) -> DeviceCSR:
+    """C = A*B for CSR matrices on the GPU (sorted columns, structural zeros kept)."""
+    with SpGEMM(A, B, validate=validate, stream=stream) as op:
+        op.symbolic(stream)
+        C = op.numeric(stream=stream)
+        op.wait(stream)
+    return C

@@ -1,0 +1,243 @@
+"""GPU parity against the CPU oracle on small and adversarial inputs (through the C ABI).
+
+Structure (rowptr, colidx) must be bit-exact; values within max relative
+error 1e-12 (float64) or 1e-5 (float32) of the summation-order bound.
+"""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+from synth import HostCSR, random_csr, rmat_pattern, uniform_csr
+from tests._gpu import assert_matches_oracle, run_gpu, tuning
+
+pytestmark = pytest.mark.gpu
+
+DTYPES = [np.float64, np.float32]
+
+
+def _csr(m, n, rows_cols, vals=None, dtype=np.float64):
+    rowptr = np.zeros(m + 1, dtype=np.int64)
+    cols = []
+    for i in range(m):
+        c = sorted(set(rows_cols.get(i, [])))
+        cols.extend(c)
+        rowptr[i + 1] = len(cols)
+    colidx = np.array(cols, dtype=np.int32)
+    v = np.ones(colidx.size, dtype=dtype) if vals is None else np.asarray(vals, dtype=dtype)
+    return HostCSR(m, n, rowptr, colidx, v)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("seed", range(12))
+def test_random_shapes(seed, dtype):
+    rng = np.random.default_rng(500 + seed)
+    m, k, n = (int(x) for x in rng.integers(1, 400, size=3))
+    A = random_csr(m, k, float(rng.choice([0.005, 0.02, 0.08])), rng, dtype, "sym", empty_rows=0.1)
+    B = random_csr(k, n, float(rng.choice([0.01, 0.05, 0.2])), rng, dtype, "sym", empty_rows=0.1)
+    rowptr, colidx, vals, _ = run_gpu(A, B, validate=True)
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_uniform_several_tiles(dtype):
+    # enough rows for many CTAs and a ragged last tile of every kernel
+    rng = np.random.default_rng(7)
+    A = uniform_csr(40_003, 3_001, 9, rng, dtype, "sym")
+    B = uniform_csr(3_001, 5_003, 17, rng, dtype, "sym")
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["hash_rows"] == 40_003
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_every_row_class(dtype):
+    """Rows whose product counts span every hash bin, the dense window and the direct path."""
+    rng = np.random.default_rng(11)
+    k, n = 3000, 70_000
+    B = uniform_csr(k, n, 40, rng, dtype, "sym")
+    lens = [0, 1, 1, 2, 3, 5, 9, 17, 33, 65, 100, 150, 200, 400, 1000, 2000, 3000]
+    rows = {}
+    for i, L in enumerate(lens * 3):
+        rows[i] = rng.choice(k, size=L, replace=False).tolist()
+    A = _csr(len(lens) * 3, k, rows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B, validate=True)
+    assert info["direct_rows"] == 6 and info["empty_rows"] == 3 and info["dense_rows"] > 0
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_dense_window_path_everywhere(dtype):
+    rng = np.random.default_rng(12)
+    A = uniform_csr(3000, 800, 6, rng, dtype, "sym")
+    B = uniform_csr(800, 9000, 12, rng, dtype, "sym")
+    with tuning(hash_max_products=0, dense_width=1024):
+        rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["hash_rows"] == 0 and info["dense_rows"] == 3000 and info["dense_slices"] > 3000
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_sort_path_everywhere(dtype):
+    rng = np.random.default_rng(13)
+    A = uniform_csr(2000, 900, 8, rng, dtype, "sym")
+    B = uniform_csr(900, 4000, 20, rng, dtype, "sym")
+    with tuning(run_limit=1):
+        rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["sorted_rows"] > 0
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+def test_skewed_rmat_square():
+    rng = np.random.default_rng(14)
+    rp, ci, _ = rmat_pattern(12, 16, (0.57, 0.19, 0.19, 0.05), rng)
+    A = HostCSR(4096, 4096, rp, ci, (1.0 - rng.random(ci.size)))
+    rowptr, colidx, vals, info = run_gpu(A, A)
+    assert info["dense_rows"] > 0
+    assert_matches_oracle(A, A, rowptr, colidx, vals)
+
+
+def test_rmat_unit_values_exact():
+    rng = np.random.default_rng(15)
+    rp, ci, _ = rmat_pattern(11, 16, (0.57, 0.19, 0.19, 0.05), rng)
+    A = HostCSR(2048, 2048, rp, ci, np.ones(ci.size))
+    rowptr, colidx, vals, _ = run_gpu(A, A)
+    err = assert_matches_oracle(A, A, rowptr, colidx, vals)
+    assert err == 0.0  # path counts are exact integers in any summation order
+
+
+@pytest.mark.parametrize("m,k,n", [(0, 5, 3), (4, 0, 3), (4, 5, 0), (1, 1, 1), (7, 3, 1)])
+def test_degenerate_shapes(m, k, n):
+    rng = np.random.default_rng(m * 100 + k * 10 + n)
+    A = random_csr(m, k, 0.6, rng)
+    B = random_csr(k, n, 0.6, rng)
+    rowptr, colidx, vals, _ = run_gpu(A, B, validate=True)
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+def test_all_rows_empty_and_empty_b_rows():
+    A = _csr(50, 20, {i: [i % 20] for i in range(0, 50, 2)})
+    B = _csr(20, 30, {j: [j, j + 1] for j in range(1, 20, 2)})  # even rows of B empty
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert rowptr[-1] == 0 and info["empty_rows"] == 50
+
+
+def test_direct_rows_scaled_copy():
+    rng = np.random.default_rng(16)
+    perm = rng.permutation(500)
+    A = HostCSR(500, 500, np.arange(501, dtype=np.int64), perm.astype(np.int32), 2 * rng.random(500) - 1)
+    B = uniform_csr(500, 2000, 37, rng)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["direct_rows"] == 500
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+def test_single_dense_row_and_wide_output():
+    rng = np.random.default_rng(17)
+    k, n = 600, 1 << 20
+    A = _csr(3, k, {0: list(range(k)), 2: [5, 7]}, dtype=np.float64)
+    A.vals = 2 * rng.random(A.nnz) - 1
+    B = uniform_csr(k, n, 30, rng)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["dense_rows"] == 1
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+def test_cancellation_keeps_structural_zero():
+    A = _csr(1, 2, {0: [0, 1]}, vals=[1.0, -1.0])
+    B = _csr(2, 3, {0: [0, 2], 1: [0, 1]}, vals=[2.0, 5.0, 2.0, 3.0])
+    rowptr, colidx, vals, _ = run_gpu(A, B)
+    assert rowptr.tolist() == [0, 3]
+    assert colidx.tolist() == [0, 1, 2]
+    assert vals.tolist() == [0.0, -3.0, 5.0]
+
+
+def test_handle_reuse_and_growth():
+    """One SpGEMM object re-run, then a second, larger product: scratch grows, results stay exact."""
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+    rng = np.random.default_rng(18)
+    A = uniform_csr(1000, 700, 5, rng)
+    B = uniform_csr(700, 900, 7, rng)
+    dA, dB = DeviceCSR.from_host(A), DeviceCSR.from_host(B)
+    with SpGEMM(dA, dB) as op:
+        outs = []
+        for _ in range(3):
+            op.symbolic()
+            C = op.numeric()
+            op.wait()
+            outs.append(C.to_host())
+    for o in outs[1:]:
+        for a, b in zip(outs[0][:2], o[:2]):
+            np.testing.assert_array_equal(a, b)
+    assert_matches_oracle(A, B, *outs[-1])
+    A2 = uniform_csr(30_000, 700, 9, rng)
+    rowptr, colidx, vals, _ = run_gpu(A2, B)
+    assert_matches_oracle(A2, B, rowptr, colidx, vals)
+
+
+def test_device_count_check_reports_error():
+    """A row pointer altered between the passes is caught by the numeric pass's count check."""
+    from paper_2606_20855_gb300 import _abi
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+    rng = np.random.default_rng(19)
+    A = uniform_csr(256, 300, 6, rng)
+    B = uniform_csr(300, 5000, 8, rng)
+    with SpGEMM(DeviceCSR.from_host(A), DeviceCSR.from_host(B)) as op:
+        nnz = op.symbolic()
+        # move one entry from row 10 to row 11: every write stays inside [0, nnz)
+        op.c_rowptr[11] -= 1
+        C = op.numeric()
+        with pytest.raises(_abi.WsError) as ei:
+            op.wait()
+        assert ei.value.status_name == "WS_ERR_DEVICE"
+        assert C.nnz == nnz
+        # the handle stays usable
+        op.symbolic()
+        C = op.numeric()
+        op.wait()
+        rowptr, colidx, vals = C.to_host()
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+def test_host_side_errors():
+    from paper_2606_20855_gb300 import _abi
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+    rng = np.random.default_rng(20)
+    A = uniform_csr(10, 8, 3, rng)
+    B = uniform_csr(9, 8, 3, rng)
+    with pytest.raises(_abi.WsError) as ei:
+        with SpGEMM(DeviceCSR.from_host(A), DeviceCSR.from_host(B)) as op:
+            op.symbolic()
+    assert ei.value.status_name == "WS_ERR_SHAPE"
+    B32 = uniform_csr(8, 8, 3, rng, np.float32)
+    with pytest.raises(TypeError):
+        SpGEMM(DeviceCSR.from_host(A), DeviceCSR.from_host(B32))
+    # invalid CSR: unsorted columns, duplicate, out of range, non-monotone rowptr
+    good = uniform_csr(6, 10, 3, rng)
+    bads = []
+    b = HostCSR(6, 10, good.rowptr.copy(), good.colidx.copy(), good.vals.copy())
+    b.colidx[0], b.colidx[1] = b.colidx[1], b.colidx[0]
+    bads.append(b)
+    b = HostCSR(6, 10, good.rowptr.copy(), good.colidx.copy(), good.vals.copy())
+    b.colidx[4] = b.colidx[3]
+    bads.append(b)
+    b = HostCSR(6, 10, good.rowptr.copy(), good.colidx.copy(), good.vals.copy())
+    b.colidx[-1] = 10
+    bads.append(b)
+    b = HostCSR(6, 10, good.rowptr.copy(), good.colidx.copy(), good.vals.copy())
+    b.rowptr[2], b.rowptr[3] = b.rowptr[3], b.rowptr[2]
+    bads.append(b)
+    for bad in bads:
+        with pytest.raises(_abi.WsError) as ei:
+            SpGEMM(DeviceCSR.from_host(bad), DeviceCSR.from_host(uniform_csr(10, 4, 2, rng)), validate=True)
+        assert ei.value.status_name == "WS_ERR_INVALID_CSR"
+    # numeric before symbolic
+    with SpGEMM(DeviceCSR.from_host(good), DeviceCSR.from_host(uniform_csr(10, 4, 2, rng))) as op:
+        with pytest.raises(RuntimeError):
+            op.numeric()
+        h = op._hC
+        with pytest.raises(_abi.WsError) as ei:
+            _abi.ws_spgemm_numeric(op._hA, op._hB, h, 0, 0, torch.cuda.current_stream().cuda_stream)
+        assert ei.value.status_name == "WS_ERR_STATE"
