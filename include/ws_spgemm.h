@@ -155,8 +155,8 @@ ws_status_t ws_csr_nnz(ws_csr_t handle, int64_t* nnz_out);
  * path, info[4] dense-window rows, info[5] dense-window slices,
  * info[6] total products (sum over rows of the product count),
  * info[7] number of kernel launches queued by the last symbolic pass,
- * info[8] number queued by the last numeric pass.
- * `n` is the length of `info` (at most 9 values are written).
+ * info[8] number queued by the last numeric pass, info[9] bitmap rows.
+ * `n` is the length of `info` (at most 10 values are written).
  */
 ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
 
@@ -169,6 +169,10 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
  *          (default 64; smaller values send more rows to the sorting path)
  *   key 3: dense-window slice width in columns (default 8192 for double,
  *          16384 for float; must be a multiple of 1024, 0 = default)
+ *   key 4: widest column range of a row that uses the bitmap path
+ *          (default and maximum 65536; 0 disables the bitmap path)
+ *   key 5: most stored A entries of a row that uses the one-warp register
+ *          bitmap path (default and maximum 16; 0 disables that path)
  * Returns WS_ERR_INVALID_ARG for an unknown key or out-of-range value.
  */
 ws_status_t ws_set_tuning(int key, int64_t value);

@@ -23,11 +23,31 @@ __device__ __forceinline__ int ceil_log2_ll(long long x) {  // x >= 1
   return x <= 1 ? 0 : 64 - __clzll(x - 1);
 }
 
-// Class and segment of a row from its stored-entry count and product count.
-__device__ __forceinline__ uint8_t classify(long long nnza, long long ub, long long hash_max) {
+// Class of a row from its stored-entry count, product count and column range.
+// Bitmap bins take rows whose range fits a bitmap that is not much larger
+// than the row's products (at most 8 words per product plus 64).
+// Rows with at most kBmrMaxA entries whose B rows fit one lane group take the
+// register bitmap bins.
+__device__ __forceinline__ uint8_t classify(long long nnza, long long ub, int lo, int hi, int maxlen,
+                                            const AnalyzeParams& ap) {
   if (ub == 0) return kClsEmpty;
   if (nnza == 1) return kClsDirect;
-  if (ub <= hash_max) {
+  const long long span = static_cast<long long>(hi) - lo + 1;
+  if (span <= ap.bitmap_span && ((span + 31) >> 5) <= 8 * ub + 64) {
+    if (nnza <= ap.bmr_max_a && maxlen <= ap.group) {
+#pragma unroll
+      for (int b = 0; b < kNumBmrBins; ++b) {
+        if (span <= (32ll << bmr_log_words(b))) return static_cast<uint8_t>(kClsBmr0 + b);
+      }
+    }
+    const long long est = ub < span ? ub : span;  // entries of the row are at most this
+#pragma unroll
+    for (int b = 0; b < kNumBitmapBins; ++b) {
+      if (span <= (32ll << bitmap_log_words(b)) && est <= bitmap_cap(b))
+        return static_cast<uint8_t>(kClsBitmap0 + b);
+    }
+  }
+  if (ub <= ap.hash_max) {
     int b = ceil_log2_ll(ub) - (kMinHashLog - 1);
     b = b < 0 ? 0 : b;
     return static_cast<uint8_t>(kClsHash0 + b);
@@ -38,14 +58,16 @@ __device__ __forceinline__ uint8_t classify(long long nnza, long long ub, long l
 __device__ __forceinline__ int segment_of(uint8_t cls) {
   if (cls == kClsDirect) return kSegDirect;
   if (cls == kClsDense) return kSegDense;
-  return kSegHash0 + (cls - kClsHash0);  // hash bins
+  if (cls < kClsBitmap0) return kSegBmr0 + (cls - kClsBmr0);      // register bitmap bins
+  if (cls < kClsHash0) return kSegBitmap0 + (cls - kClsBitmap0);  // bitmap bins
+  return kSegHash0 + (cls - kClsHash0);                            // hash bins
 }
 
 template <typename T>
 __device__ __forceinline__ void record_row(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t i, long long nnza,
-                                           long long ub, int lo, int hi, int* s_seg, long long* s_prod,
+                                           long long ub, int lo, int hi, int maxlen, int* s_seg, long long* s_prod,
                                            long long* s_slices, int* s_empty) {
-  const uint8_t c = classify(nnza, ub, ap.hash_max);
+  const uint8_t c = classify(nnza, ub, lo, hi, maxlen, ap);
   p.cls[i] = c;
   // Direct rows know their count already; the others start at 0 and are
   // filled by the hash / dense-window symbolic kernels.
@@ -101,18 +123,19 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
       continue;
     }
     long long ub = 0;
-    int lo = INT_MAX, hi = -1;
+    int lo = INT_MAX, hi = -1, maxlen = 0;
 #pragma unroll 4
     for (int64_t q = s; q < e; ++q) {
       const int k = p.A.colidx[q];
       const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];
       if (be > bs) {
         ub += be - bs;
+        maxlen = max(maxlen, static_cast<int>(min(be - bs, static_cast<int64_t>(INT_MAX))));
         lo = min(lo, p.B.colidx[bs]);
         hi = max(hi, p.B.colidx[be - 1]);
       }
     }
-    record_row(p, ap, i, e - s, ub, lo, hi, s_seg, &s_prod, &s_slices, &s_empty);
+    record_row(p, ap, i, e - s, ub, lo, hi, maxlen, s_seg, &s_prod, &s_slices, &s_empty);
   }
   __syncthreads();
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
@@ -156,7 +179,7 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
       lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
       hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
-    if (lane == 0) record_row(p, ap, i, e - s, ub, lo, hi, s_seg, &s_prod, &s_slices, &s_empty);
+    if (lane == 0) record_row(p, ap, i, e - s, ub, lo, hi, INT_MAX, s_seg, &s_prod, &s_slices, &s_empty);
   }
   __syncthreads();
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);

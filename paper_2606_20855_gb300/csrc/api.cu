@@ -27,6 +27,8 @@ thread_local std::string g_last_error;
 
 // Process-wide tuning (ws_set_tuning).
 int64_t g_hash_max = kMaxHashProducts;
+int64_t g_bitmap_span = kMaxBitmapSpan;
+int g_bmr_max_a = kBmrMaxA;
 int g_run_limit = 64;
 int g_dense_width = 0;  // 0 = default per value type
 constexpr int kLongRowThreshold = 128;
@@ -241,7 +243,8 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
 
   RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
   if (m > 0) {
-    AnalyzeParams ap{m, g_hash_max, pl->dense_width, kLongRowThreshold};
+    AnalyzeParams ap{m, g_hash_max, g_bitmap_span, 1 << pl->log2_group, g_bmr_max_a, pl->dense_width,
+                     kLongRowThreshold};
     launch_analyze<T>(p, ap, pl->long_rows, sms, s, &pl->sym_launches);
     WS_CUDA(cudaGetLastError(), "analyze launch");
   }
@@ -271,6 +274,20 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
     p.seg_len = pl->seg_count[kSegDense];
     launch_dense_slices<T>(p, pl->slice_row, pl->slice_idx, pl->slice_first, sms, s, &pl->sym_launches);
     launch_dense<T>(p, pl->dense_slices, false, sms, s, &pl->sym_launches);
+  }
+  for (int b = 0; b < kNumBmrBins; ++b) {
+    const int g = kSegBmr0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_bmr<T>(p, b, false, sms, s, &pl->sym_launches);
+  }
+  for (int b = 0; b < kNumBitmapBins; ++b) {
+    const int g = kSegBitmap0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_bitmap<T>(p, b, false, sms, s, &pl->sym_launches);
   }
   for (int b = 0; b < kNumHashBins; ++b) {
     const int g = kSegHash0 + b;
@@ -305,6 +322,20 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     p.seg_begin = pl->seg_offset[kSegDirect];
     p.seg_len = pl->seg_count[kSegDirect];
     launch_direct<T>(p, sms, s, &pl->num_launches);
+  }
+  for (int b = 0; b < kNumBmrBins; ++b) {
+    const int g = kSegBmr0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_bmr<T>(p, b, true, sms, s, &pl->num_launches);
+  }
+  for (int b = 0; b < kNumBitmapBins; ++b) {
+    const int g = kSegBitmap0 + b;
+    if (pl->seg_count[g] == 0) continue;
+    p.seg_begin = pl->seg_offset[g];
+    p.seg_len = pl->seg_count[g];
+    launch_bitmap<T>(p, b, true, sms, s, &pl->num_launches);
   }
   for (int b = 0; b < kNumHashBins; ++b) {
     const int g = kSegHash0 + b;
@@ -489,10 +520,12 @@ ws_status_t ws_csr_nnz(ws_csr_t h, int64_t* nnz_out) {
 ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
   if (!C || !info || n < 0) return fail(WS_ERR_INVALID_ARG, "NULL argument");
   const Plan* pl = C->plan;
-  int64_t v[9] = {0, 0, 0, 0, 0, 0, 0, 0, 0};
+  int64_t v[10] = {0, 0, 0, 0, 0, 0, 0, 0, 0, 0};
   if (pl) {
-    int64_t hash_rows = 0;
+    int64_t hash_rows = 0, bitmap_rows = 0;
     for (int b = 0; b < kNumHashBins; ++b) hash_rows += pl->seg_count[kSegHash0 + b];
+    for (int b = 0; b < kNumBitmapBins; ++b) bitmap_rows += pl->seg_count[kSegBitmap0 + b];
+    for (int b = 0; b < kNumBmrBins; ++b) bitmap_rows += pl->seg_count[kSegBmr0 + b];
     v[0] = pl->n_empty;
     v[1] = pl->seg_count[kSegDirect];
     v[2] = hash_rows;
@@ -502,8 +535,9 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
     v[6] = pl->products;
     v[7] = pl->sym_launches;
     v[8] = pl->num_launches;
+    v[9] = bitmap_rows;
   }
-  for (int i = 0; i < n && i < 9; ++i) info[i] = v[i];
+  for (int i = 0; i < n && i < 10; ++i) info[i] = v[i];
   return WS_OK;
 }
 
@@ -521,6 +555,14 @@ ws_status_t ws_set_tuning(int key, int64_t value) {
       if (value != 0 && (value < 1024 || value > 16384 || value % 1024 != 0))
         return fail(WS_ERR_INVALID_ARG, "dense width must be 0 or a multiple of 1024 in [1024, 16384]");
       g_dense_width = static_cast<int>(value);
+      return WS_OK;
+    case 4:
+      if (value < 0 || value > kMaxBitmapSpan) return fail(WS_ERR_INVALID_ARG, "bitmap span out of range");
+      g_bitmap_span = value;
+      return WS_OK;
+    case 5:
+      if (value < 0 || value > kBmrMaxA) return fail(WS_ERR_INVALID_ARG, "register-row entry limit out of range");
+      g_bmr_max_a = static_cast<int>(value);
       return WS_OK;
   }
   return fail(WS_ERR_INVALID_ARG, "unknown tuning key %d", key);

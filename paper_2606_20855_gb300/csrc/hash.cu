@@ -24,8 +24,10 @@
 // insertion order, so the numeric pass (same keys, same table, same hash)
 // sees exactly the clusters the symbolic pass checked.
 //
-// Table sizes: bin b holds rows with at most 32 << b products in 64 << b
-// slots, so the load factor is at most 1/2.
+// Table sizes: bin b holds rows with at most 32 << b products whose home
+// slots span 64 << b slots, so the load factor is at most 1/2.  The table
+// has tail_slots() extra slots past the home range, so a run of keys that reaches
+// the end of the home range continues upward instead of wrapping to slot 0.
 #include "ws_internal.cuh"
 
 namespace wsk {
@@ -33,7 +35,11 @@ namespace wsk {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kUnroll = 4;  // B entries a lane loads before inserting them
 constexpr int kEmptyKey = -1;
+// Slots past the home range: at least 64, and a multiple of 32 per warp so
+// every warp of a row team ranks a whole number of 32-slot chunks.
+__host__ __device__ constexpr int tail_slots(int wpr) { return 32 * (wpr > 2 ? wpr : 2); }
 
 template <int WPR>
 __device__ __forceinline__ void team_sync() {
@@ -49,29 +55,33 @@ __device__ __forceinline__ void atomic_add_value(T* addr, T v) {
   atomicAdd(addr, v);
 }
 
-// Inserts key c (and adds v when NUMERIC) into the table; returns 1 if the
-// key was new, 0 if it was present, -1 if the whole table was probed.
+// Inserts key c (and adds v when NUMERIC) into the table.  Returns a bit set:
+// kInsNew if the key was new, kInsWrapped if the probe wrapped from the last
+// slot to slot 0, kInsFailed if every slot was probed.
+constexpr int kInsNew = 1, kInsWrapped = 2, kInsFailed = 4;
 template <bool NUMERIC, typename T>
-__device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint32_t mask, int c, T v,
-                                            bool& wrapped) {
+__device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint32_t nslots, int c, T v) {
   volatile int* vk = keys;
-  for (uint32_t n = 0; n <= mask; ++n) {
+  int wrapped = 0;
+  for (uint32_t n = 0; n < nslots; ++n) {
     int cur = vk[h];
     if (cur == kEmptyKey) {
       cur = atomicCAS(&keys[h], kEmptyKey, c);
       if (cur == kEmptyKey) {
         if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
-        return 1;
+        return kInsNew | wrapped;
       }
     }
     if (cur == c) {
       if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
-      return 0;
+      return wrapped;
     }
-    h = (h + 1) & mask;
-    wrapped |= (h == 0);
+    if (++h == nslots) {
+      h = 0;
+      wrapped = kInsWrapped;
+    }
   }
-  return -1;
+  return kInsFailed | wrapped;
 }
 
 // True if the table holds a run of more than `limit` occupied slots.  Called
@@ -105,23 +115,26 @@ __device__ __forceinline__ void clear_values(T* vals, int n, int t, int nt) {
 }
 
 // LOGT: log2 of table slots; WPR: warps per row team; RPC: row teams per CTA.
+// The launch bounds let the compiler use up to 64 registers per thread.
 template <typename T, int LOGT, int WPR, int RPC, bool NUMERIC>
-__global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan<T> p, const uint8_t my_cls) {
+__global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_rows_kernel(const RowPlan<T> p, const uint8_t my_cls) {
   static_assert(WPR == 1 || RPC == 1, "multi-warp row teams use the whole CTA");
-  constexpr int kT = 1 << LOGT;
-  constexpr uint32_t kMask = kT - 1;
+  constexpr int kT = 1 << LOGT;        // home range
+  constexpr int kS = kT + tail_slots(WPR);  // slots
   constexpr int kNT = 32 * WPR;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int s_warp[WPR > 1 ? WPR : 1];
   __shared__ int s_flags;
+  __shared__ long long s_b0[kNT * RPC], s_b1[kNT * RPC];  // staged B-row bounds of A entries
+  __shared__ T s_a[kNT * RPC];                             // staged A values
 
   const int sub = threadIdx.x / kNT;
   const int t = threadIdx.x % kNT;
   const int lane = threadIdx.x & 31;
   const int warp = t >> 5;
-  int* keys = reinterpret_cast<int*>(smem_raw) + sub * kT;
+  int* keys = reinterpret_cast<int*>(smem_raw) + sub * kS;
   T* vals = nullptr;
-  if constexpr (NUMERIC) vals = reinterpret_cast<T*>(reinterpret_cast<int*>(smem_raw) + RPC * kT) + sub * kT;
+  if constexpr (NUMERIC) vals = reinterpret_cast<T*>(reinterpret_cast<int*>(smem_raw) + RPC * kS) + sub * kS;
 
   const int lg = p.log2_group;
   const int gsize = 1 << lg;
@@ -143,8 +156,8 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
     // Clear the workspace (w .= 0).
     {
       int4* k4 = reinterpret_cast<int4*>(keys);
-      for (int s = t; s < kT / 4; s += kNT) k4[s] = make_int4(kEmptyKey, kEmptyKey, kEmptyKey, kEmptyKey);
-      if constexpr (NUMERIC) clear_values(vals, kT, t, kNT);
+      for (int s = t; s < kS / 4; s += kNT) k4[s] = make_int4(kEmptyKey, kEmptyKey, kEmptyKey, kEmptyKey);
+      if constexpr (NUMERIC) clear_values(vals, kS, t, kNT);
       if constexpr (WPR > 1) {
         if (t < WPR) s_warp[t] = 0;
         if (t == 0) s_flags = 0;
@@ -153,25 +166,69 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
     team_sync<WPR>();
 
     // Accumulate: w[j] += A[i,k] * B[k,j] for every stored A[i,k], B[k,j].
-    int my_new = 0;
-    bool wrapped = false, failed = false;
-    const int64_t pa_end = p.A.rowptr[row + 1];
-    for (int64_t pa = p.A.rowptr[row] + grp; pa < pa_end; pa += ngrp) {
-      const int k = p.A.colidx[pa];
-      T av = T(0);
-      if constexpr (NUMERIC) av = p.A.vals[pa];
-      const int64_t qe = p.B.rowptr[k + 1];
-      for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
-        const int c = p.B.colidx[q];
-        T v = T(0);
-        if constexpr (NUMERIC) v = av * p.B.vals[q];
-        const uint32_t d = static_cast<uint32_t>(c - lo);
-        const uint32_t h = ident ? d : static_cast<uint32_t>((static_cast<unsigned long long>(d) * mul) >> 32);
-        const int res = probe_insert<NUMERIC>(keys, vals, h, kMask, c, v, wrapped);
-        my_new += res > 0;
-        failed |= res < 0;
+    // The team first stages a chunk of the row's A entries (B-row bounds and
+    // A values) in shared memory, then every group of gsize lanes walks B
+    // rows, loading kUnroll B entries before it inserts any of them.
+    int my_new = 0, my_flags = 0;
+#define WS_INSERT(c_, v_)                                                                                     \
+  do {                                                                                                        \
+    const uint32_t d_ = static_cast<uint32_t>((c_) - lo);                                                     \
+    const uint32_t h_ = ident ? d_ : static_cast<uint32_t>((static_cast<unsigned long long>(d_) * mul) >> 32); \
+    const int r_ = probe_insert<NUMERIC>(keys, vals, h_, kS, (c_), (v_));                                     \
+    my_new += r_ & kInsNew;                                                                                   \
+    my_flags |= r_;                                                                                           \
+  } while (0)
+    long long* st_b0 = s_b0 + sub * kNT;
+    long long* st_b1 = s_b1 + sub * kNT;
+    T* st_a = s_a + sub * kNT;
+    const int64_t ra = p.A.rowptr[row], re = p.A.rowptr[row + 1];
+    for (int64_t cb = ra; cb < re; cb += kNT) {
+      const int n = static_cast<int>(min(static_cast<int64_t>(kNT), re - cb));
+      if (t < n) {
+        const int k = p.A.colidx[cb + t];
+        st_b0[t] = p.B.rowptr[k];
+        st_b1[t] = p.B.rowptr[k + 1];
+        if constexpr (NUMERIC) st_a[t] = p.A.vals[cb + t];
       }
+      team_sync<WPR>();
+      for (int j0 = grp; j0 < n; j0 += ngrp * kUnroll) {
+        int cc[kUnroll];
+        T vv[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          const int j = j0 + u * ngrp;
+          cc[u] = -1;
+          vv[u] = T(0);
+          if (j < n) {
+            const long long q = st_b0[j] + gl;
+            if (q < st_b1[j]) {
+              cc[u] = p.B.colidx[q];
+              if constexpr (NUMERIC) vv[u] = st_a[j] * p.B.vals[q];
+            }
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          if (cc[u] >= 0) WS_INSERT(cc[u], vv[u]);
+        }
+        // B rows longer than the group: the rest of each row.
+#pragma unroll 1
+        for (int u = 0; u < kUnroll; ++u) {
+          const int j = j0 + u * ngrp;
+          if (j >= n) break;
+          const long long qe = st_b1[j];
+          for (long long q = st_b0[j] + gl + gsize; q < qe; q += gsize) {
+            T v = T(0);
+            if constexpr (NUMERIC) v = st_a[j] * p.B.vals[q];
+            WS_INSERT(p.B.colidx[q], v);
+          }
+        }
+      }
+      team_sync<WPR>();
     }
+#undef WS_INSERT
+    const bool wrapped = (my_flags & kInsWrapped) != 0;
+    const bool failed = (my_flags & kInsFailed) != 0;
 
     if constexpr (!NUMERIC) {
       // Count the distinct columns, check the table for the ranking condition.
@@ -192,7 +249,7 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
           total = s_warp[0];
           fl = s_flags;
         }
-        const bool long_run = has_long_run(keys, kT, p.run_limit, lane);
+        const bool long_run = has_long_run(keys, kS, p.run_limit, lane);
         if (lane == 0) {
           p.c_rowptr[row + 1] = total;
           if (fl & 2) atomicOr(&p.sum->status, kErrProbe);
@@ -206,7 +263,8 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
     } else {
       team_sync<WPR>();
       // Rank and write: each warp ranks a contiguous range of slots.
-      constexpr int kPerWarp = kT / WPR;
+      constexpr int kPerWarp = kS / WPR;
+      static_assert(kPerWarp % 32 == 0 && kPerWarp * WPR == kS, "whole chunks per warp");
       const int s_begin = warp * kPerWarp;
       int carry = 0;
       if constexpr (WPR > 1) {
@@ -241,12 +299,12 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
           }
           if (cs > 0 && steps == limit && keys[cs - 1] != kEmptyKey) rank_err = true;
           int u = s + 1;
-          for (steps = 0; u < kT && steps < limit; ++u, ++steps) {
+          for (steps = 0; u < kS && steps < limit; ++u, ++steps) {
             const int kk = keys[u];
             if (kk == kEmptyKey) break;
             rk += kk < key;
           }
-          if (u < kT && steps == limit && keys[u] != kEmptyKey) rank_err = true;
+          if (u < kS && steps == limit && keys[u] != kEmptyKey) rank_err = true;
           const int64_t pos = static_cast<int64_t>(before) - (s - cs) + rk;
           if (pos >= 0 && pos < cnt) {
             p.c_colidx[base + pos] = key;
@@ -270,8 +328,8 @@ __global__ void __launch_bounds__(32 * WPR * RPC) hash_rows_kernel(const RowPlan
 
 template <typename T, int LOGT, int WPR, int RPC>
 void launch_bin(const RowPlan<T>& p, bool numeric, int bin, int num_sms, cudaStream_t s) {
-  constexpr int kT = 1 << LOGT;
-  const size_t smem = static_cast<size_t>(RPC) * kT * (sizeof(int) + (numeric ? sizeof(T) : 0));
+  constexpr int kS = (1 << LOGT) + tail_slots(WPR);
+  const size_t smem = static_cast<size_t>(RPC) * kS * (sizeof(int) + (numeric ? sizeof(T) : 0));
   const int threads = 32 * WPR * RPC;
   auto kern = numeric ? hash_rows_kernel<T, LOGT, WPR, RPC, true> : hash_rows_kernel<T, LOGT, WPR, RPC, false>;
   static bool configured[2] = {false, false};

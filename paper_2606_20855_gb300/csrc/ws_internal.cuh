@@ -6,6 +6,8 @@
 // the load-balance problem of Sec. 1):
 //   empty         ub_i = 0                       -> no output
 //   direct        exactly one stored A[i,k]      -> C[i,:] = A[i,k] * B[k,:]
+//   bitmap bin b  column range of the row at most 32 << log_words(b) columns and
+//                 min(ub_i, range) <= cap(b)     -> bitmap + rank workspace
 //   hash bin b    ub_i <= 32 << b (b = 0..7)     -> shared-memory hash workspace of
 //                                                  64 << b slots, sort-free ranking
 //   sort          a hash row whose table showed a long run of occupied slots
@@ -27,16 +29,46 @@ constexpr int kNumHashBins = 8;
 constexpr int kMinHashLog = 6;  // bin b uses a table of 1 << (kMinHashLog + b) slots
 constexpr int kMaxHashProducts = 32 << (kNumHashBins - 1);  // 4096
 
+// Bitmap bins: bitmap of 1 << log_words 32-bit words (the row's column range
+// is at most 32 << log_words columns) and a staging array of cap entries.
+struct BitmapBin {
+  int log_words;
+  int cap;
+};
+constexpr int kNumBitmapBins = 5;
+constexpr BitmapBin kBitmapBins[kNumBitmapBins] = {{6, 256}, {9, 512}, {11, 512}, {11, 1024}, {11, 8192}};
+constexpr int kMaxBitmapSpan = 32 << 11;  // 65,536 columns
+__host__ __device__ constexpr int bitmap_log_words(int b) {
+  return b == 0 ? kBitmapBins[0].log_words : b == 1 ? kBitmapBins[1].log_words : b == 2 ? kBitmapBins[2].log_words
+       : b == 3 ? kBitmapBins[3].log_words : kBitmapBins[4].log_words;
+}
+__host__ __device__ constexpr int bitmap_cap(int b) {
+  return b == 0 ? kBitmapBins[0].cap : b == 1 ? kBitmapBins[1].cap : b == 2 ? kBitmapBins[2].cap
+       : b == 3 ? kBitmapBins[3].cap : kBitmapBins[4].cap;
+}
+
+// Register bitmap bins: rows with at most kBmrMaxA stored A entries whose B
+// rows fit one lane group; bitmap of 1 << kBmrLogWords[b] words.
+constexpr int kNumBmrBins = 3;
+constexpr int kBmrMaxA = 16;
+constexpr int kBmrCap = 512;  // >= kBmrMaxA * 32 products
+__host__ __device__ constexpr int bmr_log_words(int b) { return b == 0 ? 6 : b == 1 ? 9 : 11; }
+
 // Row class codes stored per row (uint8).
 constexpr uint8_t kClsEmpty = 0;
 constexpr uint8_t kClsDirect = 1;
-constexpr uint8_t kClsHash0 = 2;  // 2 .. 2 + kNumHashBins - 1
+constexpr uint8_t kClsBmr0 = 2;                            // .. + kNumBmrBins - 1
+constexpr uint8_t kClsBitmap0 = kClsBmr0 + kNumBmrBins;    // .. + kNumBitmapBins - 1
+constexpr uint8_t kClsHash0 = kClsBitmap0 + kNumBitmapBins;  // .. + kNumHashBins - 1
 constexpr uint8_t kClsDense = kClsHash0 + kNumHashBins;
 constexpr uint8_t kClsSort = kClsDense + 1;
 
-// Segments of the row permutation: direct rows, hash bins, dense-window rows.
+// Segments of the row permutation: direct rows, register bitmap bins, bitmap
+// bins, hash bins, dense-window rows.
 constexpr int kSegDirect = 0;
-constexpr int kSegHash0 = 1;
+constexpr int kSegBmr0 = 1;
+constexpr int kSegBitmap0 = kSegBmr0 + kNumBmrBins;
+constexpr int kSegHash0 = kSegBitmap0 + kNumBitmapBins;
 constexpr int kSegDense = kSegHash0 + kNumHashBins;
 constexpr int kNumSegs = kSegDense + 1;
 
@@ -101,7 +133,10 @@ struct RowPlan {
 // Host-side launchers (one translation unit each).
 struct AnalyzeParams {
   int64_t m;
-  int64_t hash_max;  // largest ub that uses a hash bin
+  int64_t hash_max;    // largest ub that uses a hash bin
+  int64_t bitmap_span; // largest column range that uses a bitmap bin (0: none)
+  int group;           // lanes per stored A entry in the register bitmap kernels
+  int bmr_max_a;       // most stored A entries of a register bitmap row (0: none)
   int dense_width;
   int long_threshold;
 };
@@ -116,6 +151,10 @@ void launch_dense_slices(const RowPlan<T>& p, int32_t* slice_row, int32_t* slice
                          int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_hash(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_bmr(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_bitmap(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_dense(const RowPlan<T>& p, int64_t nslices, bool numeric, int num_sms, cudaStream_t s,
                   int* launches);

@@ -76,12 +76,13 @@ def test_host_argument_errors(lib):
 
 def test_tuning_knob_validation(lib):
     try:
-        for key, bad in [(1, -1), (1, 5000), (2, 0), (3, 1000), (3, 20480), (9, 1)]:
+        for key, bad in [(1, -1), (1, 5000), (2, 0), (3, 1000), (3, 20480), (4, -1), (4, 65537), (5, 17), (9, 1)]:
             with pytest.raises(_abi.WsError):
                 _abi.ws_set_tuning(key, bad)
         _abi.ws_set_tuning("hash_max_products", 0)
         _abi.ws_set_tuning("run_limit", 8)
         _abi.ws_set_tuning("dense_width", 2048)
+        _abi.ws_set_tuning("bitmap_span", 0)
     finally:
         for k, v in _abi.TUNING_DEFAULTS.items():
             _abi.ws_set_tuning(k, v)

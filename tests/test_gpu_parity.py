@@ -29,25 +29,48 @@ def _csr(m, n, rows_cols, vals=None, dtype=np.float64):
     return HostCSR(m, n, rowptr, colidx, v)
 
 
+PATHS = {"bitmap": {}, "bitmap_generic": {"register_rows_max_a": 0}, "hash": {"bitmap_span": 0}}
+
+
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("dtype", DTYPES)
 @pytest.mark.parametrize("seed", range(12))
-def test_random_shapes(seed, dtype):
+def test_random_shapes(seed, dtype, path):
     rng = np.random.default_rng(500 + seed)
     m, k, n = (int(x) for x in rng.integers(1, 400, size=3))
     A = random_csr(m, k, float(rng.choice([0.005, 0.02, 0.08])), rng, dtype, "sym", empty_rows=0.1)
     B = random_csr(k, n, float(rng.choice([0.01, 0.05, 0.2])), rng, dtype, "sym", empty_rows=0.1)
-    rowptr, colidx, vals, _ = run_gpu(A, B, validate=True)
+    with tuning(**PATHS[path]):
+        rowptr, colidx, vals, _ = run_gpu(A, B, validate=True)
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("dtype", DTYPES)
-def test_uniform_several_tiles(dtype):
+def test_uniform_several_tiles(dtype, path):
     # enough rows for many CTAs and a ragged last tile of every kernel
     rng = np.random.default_rng(7)
     A = uniform_csr(40_003, 3_001, 9, rng, dtype, "sym")
     B = uniform_csr(3_001, 5_003, 17, rng, dtype, "sym")
+    with tuning(**PATHS[path]):
+        rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info[f"{path.split('_')[0]}_rows"] == 40_003
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("n", [2_000, 16_000, 60_000])
+def test_bitmap_bins(dtype, n):
+    """Rows of every bitmap bin: narrow and wide column ranges, small and large rows."""
+    rng = np.random.default_rng(n)
+    k = 2500
+    B = uniform_csr(k, n, 24, rng, dtype, "sym")
+    lens = [2, 3, 6, 11, 20, 40, 90, 200, 330]
+    rows = {i: rng.choice(k, size=L, replace=False).tolist() for i, L in enumerate(lens * 20)}
+    A = _csr(len(lens) * 20, k, rows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
     rowptr, colidx, vals, info = run_gpu(A, B)
-    assert info["hash_rows"] == 40_003
+    assert info["bitmap_rows"] > 0
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
@@ -73,7 +96,7 @@ def test_dense_window_path_everywhere(dtype):
     rng = np.random.default_rng(12)
     A = uniform_csr(3000, 800, 6, rng, dtype, "sym")
     B = uniform_csr(800, 9000, 12, rng, dtype, "sym")
-    with tuning(hash_max_products=0, dense_width=1024):
+    with tuning(hash_max_products=0, dense_width=1024, bitmap_span=0):
         rowptr, colidx, vals, info = run_gpu(A, B)
     assert info["hash_rows"] == 0 and info["dense_rows"] == 3000 and info["dense_slices"] > 3000
     assert_matches_oracle(A, B, rowptr, colidx, vals)
@@ -84,18 +107,23 @@ def test_sort_path_everywhere(dtype):
     rng = np.random.default_rng(13)
     A = uniform_csr(2000, 900, 8, rng, dtype, "sym")
     B = uniform_csr(900, 4000, 20, rng, dtype, "sym")
-    with tuning(run_limit=1):
+    with tuning(run_limit=1, bitmap_span=0):
         rowptr, colidx, vals, info = run_gpu(A, B)
     assert info["sorted_rows"] > 0
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
-def test_skewed_rmat_square():
+@pytest.mark.parametrize("path", list(PATHS))
+def test_skewed_rmat_square(path):
     rng = np.random.default_rng(14)
     rp, ci, _ = rmat_pattern(12, 16, (0.57, 0.19, 0.19, 0.05), rng)
     A = HostCSR(4096, 4096, rp, ci, (1.0 - rng.random(ci.size)))
-    rowptr, colidx, vals, info = run_gpu(A, A)
-    assert info["dense_rows"] > 0
+    with tuning(**PATHS[path]):
+        rowptr, colidx, vals, info = run_gpu(A, A)
+    if path == "hash":
+        assert info["dense_rows"] > 0 and info["bitmap_rows"] == 0
+    else:
+        assert info["bitmap_rows"] > 0
     assert_matches_oracle(A, A, rowptr, colidx, vals)
 
 
