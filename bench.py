@@ -176,12 +176,21 @@ def barrier(world: int, pg) -> None:
         pg.barrier()
 
 
+def load_workload(args):
+    """The named workload, optionally cut to the first --rows rows of A."""
+    A, B = workload(args.workload)
+    if args.rows and args.rows < A.nrows:
+        from synth import row_subset
+        A = row_subset(A, np.arange(args.rows))  # B stays the full right operand
+    return A, B
+
+
 def run_reference(args, world, rank) -> None:
     """CPU oracle arm: each step computes a bounded row sample on the host cores."""
     if rank != 0:
         return
     from oracle import oracle_spgemm
-    A, B = workload(args.workload)
+    A, B = load_workload(args)
     ub = products_per_row(A, B)
     cores = os.cpu_count() or 1
     rng = np.random.default_rng(1234)
@@ -222,7 +231,7 @@ def run_ours(args, world, rank, local, pg) -> None:
     _abi.load()
     device = torch.device(f"cuda:{local}")
     torch.cuda.set_device(device)
-    A, B = workload(args.workload)
+    A, B = load_workload(args)
     same = B is A
     ub = products_per_row(A, B)
     products = int(ub.sum())
@@ -330,7 +339,8 @@ def run_ours(args, world, rank, local, pg) -> None:
         "dtype": "f64" if s == 8 else "f32",
         "data": "synthetic",
         "config": {
-            "workload": args.workload, "description": WORKLOADS[args.workload],
+            "workload": args.workload if not args.rows else f"{args.workload}[:{A.nrows} rows]",
+            "description": WORKLOADS[args.workload],
             "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_a": A.nnz, "nnz_b": B.nnz, "nnz_c": int(nnz),
             "products": products, "l2": "flushed between timed steps (write of a buffer > L2)",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
@@ -364,6 +374,8 @@ def main(argv=None) -> int:
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
     ap.add_argument("--ref-step-s", type=float, default=4.0, help="seconds per reference-arm step")
+    ap.add_argument("--rows", type=int, default=0,
+                    help="use only the first ROWS rows of A (a smaller case of the same workload, for profiling)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu DRAM bytes per numeric launch, when captured for the current kernels")
     args = ap.parse_args(argv)

@@ -58,6 +58,7 @@ __device__ __forceinline__ uint8_t classify(long long nnza, long long ub, int lo
 __device__ __forceinline__ int segment_of(uint8_t cls) {
   if (cls == kClsDirect) return kSegDirect;
   if (cls == kClsDense) return kSegDense;
+  if (cls == kClsBmrWide) return kSegBmrWide;
   if (cls < kClsBitmap0) return kSegBmr0 + (cls - kClsBmr0);      // register bitmap bins
   if (cls < kClsHash0) return kSegBitmap0 + (cls - kClsBitmap0);  // bitmap bins
   return kSegHash0 + (cls - kClsHash0);                            // hash bins
@@ -104,7 +105,7 @@ __device__ __forceinline__ void flush_counts(const RowPlan<T>& p, int* s_seg, lo
 // longer rows are queued for analyze_long_kernel.
 template <typename T>
 __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const AnalyzeParams ap,
-                                                      int32_t* long_rows) {
+                                                      int32_t* long_rows, const int32_t* rows) {
   __shared__ int s_seg[kNumSegs];
   __shared__ long long s_prod, s_slices;
   __shared__ int s_empty;
@@ -115,8 +116,10 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
     s_empty = 0;
   }
   __syncthreads();
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < ap.m;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  const int64_t nrows = rows ? static_cast<int64_t>(*reinterpret_cast<volatile int*>(&p.sum->n_pending)) : ap.m;
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < nrows;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t i = rows ? rows[t] : t;
     const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
     if (e - s > ap.long_threshold) {
       long_rows[atomicAdd(&p.sum->n_long, 1)] = static_cast<int32_t>(i);
@@ -273,9 +276,9 @@ int grid_for(int64_t work, int per_block, int num_sms, int blocks_per_sm) {
 }  // namespace
 
 template <typename T>
-void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, int num_sms,
-                    cudaStream_t s, int* launches) {
-  analyze_kernel<T><<<grid_for(ap.m, 256, num_sms, 8), 256, 0, s>>>(p, ap, long_rows);
+void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, const int32_t* rows,
+                    int num_sms, cudaStream_t s, int* launches) {
+  analyze_kernel<T><<<grid_for(ap.m, 256, num_sms, 8), 256, 0, s>>>(p, ap, long_rows, rows);
   analyze_long_kernel<T><<<num_sms * 2, 256, 0, s>>>(p, ap, long_rows);
   *launches += 2;
 }
@@ -303,7 +306,8 @@ void launch_validate(const int64_t* rowptr, const int32_t* colidx, int64_t nrows
 }
 
 #define WS_INST(T)                                                                                          \
-  template void launch_analyze<T>(const RowPlan<T>&, const AnalyzeParams&, int32_t*, int, cudaStream_t, int*); \
+  template void launch_analyze<T>(const RowPlan<T>&, const AnalyzeParams&, int32_t*, const int32_t*, int,      \
+                                  cudaStream_t, int*);                                                       \
   template void launch_scatter<T>(const RowPlan<T>&, int64_t, const int64_t*, int, cudaStream_t, int*);      \
   template void launch_dense_slices<T>(const RowPlan<T>&, int32_t*, int32_t*, int32_t*, int, cudaStream_t, int*);
 WS_INST(float)

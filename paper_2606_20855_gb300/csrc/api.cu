@@ -87,6 +87,7 @@ struct DevBuf {
 struct Plan {
   DevBuf rows;    // per-row arrays + summary + scan partials
   DevBuf slices;  // dense-window slice arrays
+  DevBuf ranks;   // register bitmap rows: kBmrSlots uint16 ranks per row of A
   DevSummary* host_sum = nullptr;  // pinned
   // carved pointers
   DevSummary* dsum = nullptr;
@@ -96,6 +97,7 @@ struct Plan {
   int32_t* hi = nullptr;
   int32_t* long_rows = nullptr;
   int32_t* sort_list = nullptr;
+  int32_t* pending = nullptr;
   int64_t* partials = nullptr;
   int32_t* slice_row = nullptr;
   int32_t* slice_idx = nullptr;
@@ -110,6 +112,7 @@ struct Plan {
   int64_t seg_offset[kNumSegs + 1] = {};
   int64_t n_sort = 0, n_empty = 0, dense_slices = 0, products = 0;
   int log2_group = 5;
+  int wide_bin = 2;  // register bitmap bin of the rows counted by the planning pass
   int dense_width = 0;
   int run_limit = 64;
   int sym_launches = 0, num_launches = 0;
@@ -179,6 +182,7 @@ RowPlan<T> make_rowplan(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan*
   p.slice_idx = pl->slice_idx;
   p.slice_first = pl->slice_first;
   p.slice_cnt = pl->slice_cnt;
+  p.ranks = static_cast<uint16_t*>(pl->ranks.ptr);
   p.sum = pl->dsum;
   p.log2_group = pl->log2_group;
   p.run_limit = pl->run_limit;
@@ -195,6 +199,7 @@ ws_status_t carve_rows(Plan* pl, int64_t m, cudaStream_t s) {
   const size_t o_hi = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
   const size_t o_long = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
   const size_t o_sort = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
+  const size_t o_pend = off; off = align_up(off + 4 * static_cast<size_t>(m), 256);
   const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
   const size_t o_cls = off; off = align_up(off + static_cast<size_t>(m), 256);
   ws_status_t st = pl->rows.reserve(off, s);
@@ -206,6 +211,7 @@ ws_status_t carve_rows(Plan* pl, int64_t m, cudaStream_t s) {
   pl->hi = reinterpret_cast<int32_t*>(b + o_hi);
   pl->long_rows = reinterpret_cast<int32_t*>(b + o_long);
   pl->sort_list = reinterpret_cast<int32_t*>(b + o_sort);
+  pl->pending = reinterpret_cast<int32_t*>(b + o_pend);
   pl->partials = reinterpret_cast<int64_t*>(b + o_part);
   pl->cls = reinterpret_cast<uint8_t*>(b + o_cls);
   return WS_OK;
@@ -245,7 +251,20 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
   if (m > 0) {
     AnalyzeParams ap{m, g_hash_max, g_bitmap_span, 1 << pl->log2_group, g_bmr_max_a, pl->dense_width,
                      kLongRowThreshold};
-    launch_analyze<T>(p, ap, pl->long_rows, sms, s, &pl->sym_launches);
+    // When every row of C fits the widest register bitmap (B has at most
+    // 65,536 columns), the planning pass counts the eligible rows in its first
+    // read of A and only the remaining rows go through the analysis kernel.
+    const bool plan_pass = g_bmr_max_a > 0 && B->ncols > 0 && B->ncols <= kMaxBitmapSpan && g_bitmap_span >= B->ncols;
+    pl->wide_bin = bmr_bin_for_span(B->ncols);
+    if (plan_pass) {
+      st = pl->ranks.reserve(static_cast<size_t>(m) * kBmrSlots * sizeof(uint16_t), s);
+      if (st != WS_OK) return st;
+      p.ranks = static_cast<uint16_t*>(pl->ranks.ptr);
+      launch_bmr_plan<T>(p, ap, B->ncols, pl->pending, sms, s, &pl->sym_launches);
+      launch_analyze<T>(p, ap, pl->long_rows, pl->pending, sms, s, &pl->sym_launches);
+    } else {
+      launch_analyze<T>(p, ap, pl->long_rows, nullptr, sms, s, &pl->sym_launches);
+    }
     WS_CUDA(cudaGetLastError(), "analyze launch");
   }
   st = read_summary(pl, s);
@@ -265,6 +284,13 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
 
   if (off > 0) {
     launch_scatter<T>(p, m, pl->seg_offset, sms, s, &pl->sym_launches);
+  }
+  int64_t bmr_rows = 0;
+  for (int b = 0; b < kNumBmrBins; ++b) bmr_rows += pl->seg_count[kSegBmr0 + b];
+  if (bmr_rows > 0) {
+    st = pl->ranks.reserve(static_cast<size_t>(m) * kBmrSlots * sizeof(uint16_t), s);
+    if (st != WS_OK) return st;
+    p.ranks = static_cast<uint16_t*>(pl->ranks.ptr);
   }
   if (pl->seg_count[kSegDense] > 0) {
     st = carve_slices(pl, pl->dense_slices, s);
@@ -322,6 +348,11 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     p.seg_begin = pl->seg_offset[kSegDirect];
     p.seg_len = pl->seg_count[kSegDirect];
     launch_direct<T>(p, sms, s, &pl->num_launches);
+  }
+  if (pl->seg_count[kSegBmrWide] > 0) {
+    p.seg_begin = pl->seg_offset[kSegBmrWide];
+    p.seg_len = pl->seg_count[kSegBmrWide];
+    launch_bmr<T>(p, pl->wide_bin, true, sms, s, &pl->num_launches);
   }
   for (int b = 0; b < kNumBmrBins; ++b) {
     const int g = kSegBmr0 + b;
@@ -483,9 +514,10 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
 ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
-    if (h->plan->rows.ptr || h->plan->slices.ptr) cudaDeviceSynchronize();
+    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr) cudaDeviceSynchronize();
     h->plan->rows.release();
     h->plan->slices.release();
+    h->plan->ranks.release();
     if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
     delete h->plan;
   }
@@ -526,6 +558,7 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
     for (int b = 0; b < kNumHashBins; ++b) hash_rows += pl->seg_count[kSegHash0 + b];
     for (int b = 0; b < kNumBitmapBins; ++b) bitmap_rows += pl->seg_count[kSegBitmap0 + b];
     for (int b = 0; b < kNumBmrBins; ++b) bitmap_rows += pl->seg_count[kSegBmr0 + b];
+    bitmap_rows += pl->seg_count[kSegBmrWide];
     v[0] = pl->n_empty;
     v[1] = pl->seg_count[kSegDirect];
     v[2] = hash_rows;

@@ -1,22 +1,37 @@
 // Register bitmap rows: one warp per row for rows with at most 16 stored A
 // entries whose B rows each fit in one group of lanes (uniformly sparse
-// products such as random matrices and stencils).
+// products such as random matrices and stencils).  Every lane keeps its
+// products (column, and in the numeric pass the scaled value) in registers.
 //
-// The workspace is the bitmap + rank scheme of the bitmap rows (one bit per
-// column of the row's range, the sparse byte-map workspace of Gustavson's
-// SpGEMM, Sec. 5.1), but every lane keeps its products (column and scaled
-// value) in registers, so B is walked once per pass:
-//   symbolic:  atomicOr every product column into the bitmap and count the
-//              bits that were 0 (nnz of the row);
-//   numeric:   set the bits, rank every 128-bit chunk of the bitmap (prefix
-//              of bit counts), add each product's value at the rank of its
-//              column in a compact staging array, copy the sorted row to C.
+// Symbolic pass.  The row's workspace is a bitmap with one bit per column of
+// the row's range -- the sparse byte-map workspace of Gustavson's SpGEMM
+// (Sec. 5.1) with a bit in place of a byte.  The warp sets the bit of every
+// product column, ranks the bitmap (prefix sums of bit counts: the total is
+// nnz of the row, and the rank of a column is its position in the sorted
+// output row) and stores, for every product, the rank of its column in the
+// plan (uint16, kBmrSlots slots per row).
+// Numeric pass.  No workspace search is left: every product adds its value
+// at its stored rank in a compact staging array (a shared-memory atomic, the
+// atomic level of Sec. 4, for the rare repeated column), the column goes to
+// the same slot, and the warp copies the sorted row to C with coalesced
+// stores.  One warp owns the row (shard pattern, Sec. 4).
+//
 // Lanes are split into groups of G lanes; the group of lane l takes stored A
 // entries j = l / G, l / G + 32/G, ...; lane l takes element l % G of B[k_j,:].
+// Product (step s, lane l) has slot s * 32 + l.
 //
-// Bitmap layout: chunk i (128 bits) belongs to lane i / IPT in the rank pass
-// and is stored at i ^ ((i / IPT) & 7), so the 8 lanes of a quarter warp read
-// 8 different bank quads in every step.
+// Bitmap layout.  With WPL = words / 32 words per lane, word w is stored at
+// (w % WPL) * 32 + w / WPL: lane l owns the contiguous words [l*WPL, (l+1)*WPL)
+// and they sit in bank l.  The ranking pass reads 32 consecutive words per
+// step, and the 32 sorted columns of one B row mostly fall in different
+// banks.  After use, a row clears only the words it set.
+//
+// Planning.  When B has at most 65,536 columns every row fits the widest
+// bitmap with lo = 0, and bmr_plan_kernel handles every eligible row of A in
+// the first pass over A (no separate analysis pass for those rows); the rows
+// it does not take are queued for the analysis kernel.
+#include <climits>
+
 #include "ws_internal.cuh"
 
 namespace wsk {
@@ -29,145 +44,179 @@ constexpr int kRowsPerCta = 4;
 template <int LOGW>
 struct BmrShape {
   static constexpr int kWords = 1 << LOGW;
-  static constexpr int kChunks = kWords / 4 < 32 ? 32 : kWords / 4;
-  static constexpr int kIPT = kChunks / 32;
-  static constexpr int kLogIPT = kIPT == 1 ? 0 : kIPT == 2 ? 1 : kIPT == 4 ? 2 : kIPT == 8 ? 3 : 4;
-  static constexpr int kSwz = kIPT >= 8 ? 7 : kIPT - 1;
-  static_assert((1 << kLogIPT) == kIPT, "chunks per lane must be a power of two <= 16");
+  static constexpr int kWPL = kWords >= 32 ? kWords / 32 : 1;  // words per lane
+  static constexpr int kLogWPL = LOGW >= 5 ? LOGW - 5 : 0;
+  static constexpr int kPhysWords = kWPL * 32;
+  // symbolic: bitmap + per-word rank prefix + per-lane base; numeric: staging
   template <typename T>
   static constexpr size_t warp_bytes(bool numeric) {
-    return static_cast<size_t>(kChunks) * 16 +
-           (numeric ? static_cast<size_t>(kChunks) * 2 + 32 * 4 + static_cast<size_t>(kBmrCap) * (4 + sizeof(T)) : 0);
+    return numeric ? static_cast<size_t>(kBmrCap) * (4 + sizeof(T))
+                   : static_cast<size_t>(kPhysWords) * 6 + 32 * 4;
   }
 };
 
 template <class S>
-__device__ __forceinline__ uint32_t phys_chunk(uint32_t i) {
-  return i ^ ((i >> S::kLogIPT) & S::kSwz);
+__device__ __forceinline__ uint32_t phys_word(uint32_t w) {
+  return ((w & (S::kWPL - 1)) << 5) | (w >> S::kLogWPL);
+}
+
+// Loads the row's products into registers: lane j < na first loads stored A
+// entry j (its B row start, length and value), then every lane loads its
+// elements of the B rows of its group.
+template <typename T, int G, bool NUMERIC, int kSteps>
+__device__ __forceinline__ void load_products(const RowPlan<T>& p, int64_t ra, int na, int lane, int* col, T* val) {
+  constexpr int kGroups = 32 / G;
+  const int grp = lane / G, gl = lane % G;
+  long long my_b0 = 0;
+  int my_len = 0;
+  T my_a = T(0);
+  if (lane < na) {
+    const int k = p.A.colidx[ra + lane];
+    my_b0 = p.B.rowptr[k];
+    my_len = static_cast<int>(p.B.rowptr[k + 1] - my_b0);
+    if constexpr (NUMERIC) my_a = p.A.vals[ra + lane];
+  }
+#pragma unroll
+  for (int s = 0; s < kSteps; ++s) {
+    const int j = s * kGroups + grp;
+    const long long b0 = __shfl_sync(kFull, my_b0, j & 31);
+    const int len = __shfl_sync(kFull, my_len, j & 31);
+    T a = T(0);
+    if constexpr (NUMERIC) a = __shfl_sync(kFull, my_a, j & 31);
+    col[s] = -1;
+    val[s] = T(0);
+    if (j < na && gl < len) {
+      col[s] = p.B.colidx[b0 + gl];
+      if constexpr (NUMERIC) val[s] = a * p.B.vals[b0 + gl];
+    }
+  }
+}
+
+// Sets the bit of every product column; returns how many bits were 0 before
+// (when COUNT).  The caller clears the words after its last use.
+template <class S, bool COUNT, int kSteps>
+__device__ __forceinline__ int set_bits(uint32_t* bm, const int* col, int lo) {
+  int fresh = 0;
+#pragma unroll
+  for (int s = 0; s < kSteps; ++s) {
+    if (col[s] >= 0) {
+      const uint32_t off = static_cast<uint32_t>(col[s] - lo);
+      const uint32_t bit = 1u << (off & 31u);
+      uint32_t* word = bm + phys_word<S>(off >> 5);
+      if constexpr (COUNT) {
+        fresh += (atomicOr(word, bit) & bit) == 0u;
+      } else {
+        atomicOr(word, bit);
+      }
+    }
+  }
+  return fresh;
+}
+
+template <class S, int kSteps>
+__device__ __forceinline__ void clear_bits(uint32_t* bm, const int* col, int lo) {
+#pragma unroll
+  for (int s = 0; s < kSteps; ++s) {
+    if (col[s] >= 0) bm[phys_word<S>(static_cast<uint32_t>(col[s] - lo) >> 5)] = 0u;
+  }
+}
+
+// Ranks the row's bitmap and stores the rank of every product column at
+// ranks[s * 32 + lane]; clears the words it set; returns nnz of the row.
+template <class S, int kSteps>
+__device__ __forceinline__ int rank_products(uint32_t* bm, uint16_t* pre, int* base, const int* col, int lo, int lane,
+                                             uint16_t* ranks) {
+  set_bits<S, false, kSteps>(bm, col, lo);
+  __syncwarp();
+  int run = 0;
+#pragma unroll 8
+  for (int j = 0; j < S::kWPL; ++j) {
+    const int ph = (j << 5) | lane;
+    pre[ph] = static_cast<uint16_t>(run);
+    run += __popc(bm[ph]);
+  }
+  int incl = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += y;
+  }
+  base[lane] = incl - run;
+  const int total = __shfl_sync(kFull, incl, 31);
+  __syncwarp();
+#pragma unroll
+  for (int s = 0; s < kSteps; ++s) {
+    if (col[s] >= 0) {
+      const uint32_t off = static_cast<uint32_t>(col[s] - lo);
+      const uint32_t w = off >> 5;
+      const uint32_t ph = phys_word<S>(w);
+      const int pos = base[w >> S::kLogWPL] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
+      ranks[(s << 5) | lane] = static_cast<uint16_t>(pos);
+    }
+  }
+  __syncwarp();
+  clear_bits<S, kSteps>(bm, col, lo);
+  __syncwarp();
+  return total;
 }
 
 template <typename T, int LOGW, int G, bool NUMERIC>
-__global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 3 : 6) bmr_rows_kernel(const RowPlan<T> p) {
+__global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 5 : 6) bmr_rows_kernel(const RowPlan<T> p) {
   using S = BmrShape<LOGW>;
-  constexpr int kGroups = 32 / G;                 // A entries per step
-  constexpr int kSteps = kBmrMaxA / kGroups;       // steps that cover kBmrMaxA entries
+  constexpr int kSteps = kBmrMaxA / (32 / G);
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::template warp_bytes<T>(NUMERIC);
+  // symbolic workspace
   uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
-  uint4* bm4 = reinterpret_cast<uint4*>(ws);
-  uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kChunks) * 16);
-  int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kChunks) * 18);
-  int* st_key = base + 32;
-  T* st_val = reinterpret_cast<T*>(st_key + kBmrCap);
-  const int grp = lane / G, gl = lane % G;
+  uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
+  int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
+  // numeric workspace
+  int* st_key = reinterpret_cast<int*>(ws);
+  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kBmrCap) * 4);
+
+  if constexpr (!NUMERIC) {
+    for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
+    __syncwarp();
+  }
 
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub; r < p.seg_len;
        r += static_cast<int64_t>(gridDim.x) * kRowsPerCta) {
     const int32_t row = p.perm[p.seg_begin + r];
-    const int lo = p.lo[row];
     const int64_t ra = p.A.rowptr[row];
     const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
-    // Lane j < na holds stored A entry j: its B row start, length and value.
-    long long my_b0 = 0;
-    int my_len = 0;
-    T my_a = T(0);
-    if (lane < na) {
-      const int k = p.A.colidx[ra + lane];
-      my_b0 = p.B.rowptr[k];
-      my_len = static_cast<int>(p.B.rowptr[k + 1] - my_b0);
-      if constexpr (NUMERIC) my_a = p.A.vals[ra + lane];
-    }
-    // This lane's products: step s covers A entry s * kGroups + grp.
+    uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
     int col[kSteps];
     T val[kSteps];
-#pragma unroll
-    for (int s = 0; s < kSteps; ++s) {
-      const int j = s * kGroups + grp;
-      const long long b0 = __shfl_sync(kFull, my_b0, j & 31);
-      const int len = __shfl_sync(kFull, my_len, j & 31);
-      T a = T(0);
-      if constexpr (NUMERIC) a = __shfl_sync(kFull, my_a, j & 31);
-      col[s] = -1;
-      val[s] = T(0);
-      if (j < na && gl < len) {
-        col[s] = p.B.colidx[b0 + gl];
-        if constexpr (NUMERIC) val[s] = a * p.B.vals[b0 + gl];
-      }
-    }
-    int64_t cbase = 0;
-    int cnt = 0;
-    if constexpr (NUMERIC) {
-      cbase = p.c_rowptr[row];
-      const int64_t want = p.c_rowptr[row + 1] - cbase;
-      cnt = static_cast<int>(want < kBmrCap ? want : kBmrCap);
-      if (lane == 0 && want > kBmrCap) atomicOr(&p.sum->status, kErrCount);
-      for (int s2 = lane; s2 < cnt; s2 += 32) st_val[s2] = T(0);
-    }
-    for (int s2 = lane; s2 < S::kChunks; s2 += 32) bm4[s2] = make_uint4(0u, 0u, 0u, 0u);
-    __syncwarp();
-
-    int my_new = 0;
-#pragma unroll
-    for (int s = 0; s < kSteps; ++s) {
-      if (col[s] >= 0) {
-        const uint32_t off = static_cast<uint32_t>(col[s] - lo);
-        const uint32_t w = off >> 5;
-        const uint32_t bit = 1u << (off & 31u);
-        uint32_t* word = bm + ((phys_chunk<S>(w >> 2) << 2) | (w & 3u));
-        if constexpr (NUMERIC) {
-          atomicOr(word, bit);
-        } else {
-          my_new += (atomicOr(word, bit) & bit) == 0u;
-        }
-      }
-    }
+    load_products<T, G, NUMERIC, kSteps>(p, ra, na, lane, col, val);
 
     if constexpr (!NUMERIC) {
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) my_new += __shfl_xor_sync(kFull, my_new, o);
-      if (lane == 0) p.c_rowptr[row + 1] = my_new;
-      __syncwarp();
+      const int total = rank_products<S, kSteps>(bm, pre, base, col, p.lo[row], lane, ranks);
+      if (lane == 0) p.c_rowptr[row + 1] = total;
     } else {
-      __syncwarp();
-      // Rank of every chunk: lane l owns chunks [l * IPT, (l + 1) * IPT).
-      int run = 0;
+      int rk[kSteps];
 #pragma unroll
-      for (int j = 0; j < S::kIPT; ++j) {
-        const uint32_t ph = phys_chunk<S>(static_cast<uint32_t>(lane * S::kIPT + j));
-        const uint4 x = bm4[ph];
-        pre[ph] = static_cast<uint16_t>(run);
-        run += __popc(x.x) + __popc(x.y) + __popc(x.z) + __popc(x.w);
-      }
-      int incl = run;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += y;
-      }
-      base[lane] = incl - run;
-      const int total = __shfl_sync(kFull, incl, 31);
-      if (lane == 0 && total != cnt) atomicOr(&p.sum->status, kErrCount);
+      for (int s = 0; s < kSteps; ++s) rk[s] = col[s] >= 0 ? ranks[(s << 5) | lane] : 0;
+      const int64_t cbase = p.c_rowptr[row];
+      const int64_t want = p.c_rowptr[row + 1] - cbase;
+      const int cnt = static_cast<int>(want < kBmrCap ? want : kBmrCap);  // staging bounds every access
+      if (lane == 0 && want > kBmrCap) atomicOr(&p.sum->status, kErrCount);
+      for (int s2 = lane; s2 < cnt; s2 += 32) st_val[s2] = T(0);
       __syncwarp();
+      bool bad = false;
 #pragma unroll
       for (int s = 0; s < kSteps; ++s) {
         if (col[s] >= 0) {
-          const uint32_t off = static_cast<uint32_t>(col[s] - lo);
-          const uint32_t w = off >> 5;
-          const uint32_t i = w >> 2;
-          const uint32_t ph = phys_chunk<S>(i);
-          const uint4 x = bm4[ph];
-          const uint32_t q = w & 3u;
-          const uint32_t wd = q == 0 ? x.x : q == 1 ? x.y : q == 2 ? x.z : x.w;
-          const int pos = base[i >> S::kLogIPT] + pre[ph] + (q > 0 ? __popc(x.x) : 0) + (q > 1 ? __popc(x.y) : 0) +
-                          (q > 2 ? __popc(x.z) : 0) + __popc(wd & ((1u << (off & 31u)) - 1u));
-          if (pos < cnt) {
-            st_key[pos] = col[s];
-            atomicAdd(&st_val[pos], val[s]);
+          if (rk[s] < cnt) {
+            st_key[rk[s]] = col[s];
+            atomicAdd(&st_val[rk[s]], val[s]);
+          } else {
+            bad = true;
           }
         }
       }
+      if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
       __syncwarp();
       for (int s2 = lane; s2 < cnt; s2 += 32) {
         p.c_colidx[cbase + s2] = st_key[s2];
@@ -178,22 +227,104 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 3 : 6) bmr_rows_ke
   }
 }
 
+// First pass over A when B has at most 65,536 columns: every row with
+// 2..bmr_max_a stored entries, a non-empty product, B rows that fit one group
+// and a bitmap of at most 8 words per product is ranked right here (class
+// kClsBmrWide, lo = 0); every other row goes to `pending` for the analysis
+// kernel.  Counts per class are added to the summary.
+template <typename T, int LOGW, int G>
+__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
+                                                                   int64_t ncols, int32_t* pending) {
+  using S = BmrShape<LOGW>;
+  constexpr int kSteps = kBmrMaxA / (32 / G);
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ int s_taken;
+  __shared__ unsigned long long s_prod;
+  const int sub = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::template warp_bytes<T>(false);
+  uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
+  uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
+  int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
+  if (threadIdx.x == 0) {
+    s_taken = 0;
+    s_prod = 0;
+  }
+  for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
+  __syncthreads();
+  const long long words = (ncols + 31) >> 5;
+  int taken = 0;
+  unsigned long long prod = 0;
+
+  for (int64_t row = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub; row < ap.m;
+       row += static_cast<int64_t>(gridDim.x) * kRowsPerCta) {
+    const int64_t ra = p.A.rowptr[row];
+    const int64_t na64 = p.A.rowptr[row + 1] - ra;
+    bool ok = na64 >= 2 && na64 <= ap.bmr_max_a;
+    const int na = static_cast<int>(ok ? na64 : 0);
+    if (ok) {
+      // lane j < na: length of B row k_j
+      int my_len = 0;
+      if (lane < na) {
+        const int k = p.A.colidx[ra + lane];
+        my_len = static_cast<int>(p.B.rowptr[k + 1] - p.B.rowptr[k]);
+      }
+      int ub = my_len, mx = my_len;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        ub += __shfl_xor_sync(kFull, ub, o);
+        mx = max(mx, __shfl_xor_sync(kFull, mx, o));
+      }
+      ok = ub > 0 && mx <= G && words <= 8ll * ub + 64;
+      if (ok) {
+        int col[kSteps];
+        T unused[kSteps];
+        load_products<T, G, false, kSteps>(p, ra, na, lane, col, unused);
+        const int total = rank_products<S, kSteps>(bm, pre, base, col, 0, lane, p.ranks + row * kBmrSlots);
+        if (lane == 0) {
+          p.c_rowptr[row + 1] = total;
+          p.cls[row] = kClsBmrWide;
+          p.lo[row] = 0;
+          p.hi[row] = static_cast<int32_t>(ncols - 1);
+          ++taken;
+          prod += static_cast<unsigned long long>(ub);
+        }
+      }
+    }
+    if (!ok && lane == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
+  }
+  if (lane == 0) {
+    atomicAdd(&s_taken, taken);
+    atomicAdd(&s_prod, prod);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (s_taken) atomicAdd(&p.sum->seg_count[kSegBmrWide], s_taken);
+    if (s_prod) atomicAdd(reinterpret_cast<unsigned long long*>(&p.sum->products), s_prod);
+  }
+}
+
+template <typename K>
+int occupancy(K kern, int threads, size_t smem) {
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  int n = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, smem);
+  return n > 0 ? n : 1;
+}
+
+int64_t clamp_grid(int64_t want, int num_sms, int per_sm) {
+  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
+  return want > cap ? cap : (want < 1 ? 1 : want);
+}
+
 template <typename T, int LOGW, int G>
 void launch_bmr_g(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s) {
   using S = BmrShape<LOGW>;
   const size_t smem = static_cast<size_t>(kRowsPerCta) * S::template warp_bytes<T>(numeric);
   auto kern = numeric ? bmr_rows_kernel<T, LOGW, G, true> : bmr_rows_kernel<T, LOGW, G, false>;
   static int per_sm[2] = {0, 0};
-  if (per_sm[numeric] == 0) {
-    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    int n = 0;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, 32 * kRowsPerCta, smem);
-    per_sm[numeric] = n > 0 ? n : 1;
-  }
-  int64_t grid = (p.seg_len + kRowsPerCta - 1) / kRowsPerCta;
-  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm[numeric];
-  if (grid > cap) grid = cap;
-  if (grid < 1) grid = 1;
+  if (per_sm[numeric] == 0) per_sm[numeric] = occupancy(kern, 32 * kRowsPerCta, smem);
+  const int64_t grid = clamp_grid((p.seg_len + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm[numeric]);
   kern<<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
 }
 
@@ -205,6 +336,17 @@ void launch_bmr_w(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s
     case 4: launch_bmr_g<T, LOGW, 16>(p, numeric, num_sms, s); break;
     default: launch_bmr_g<T, LOGW, 32>(p, numeric, num_sms, s); break;
   }
+}
+
+template <typename T, int LOGW, int G>
+void launch_plan_g(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, int32_t* pending, int num_sms,
+                   cudaStream_t s) {
+  using S = BmrShape<LOGW>;
+  const size_t smem = static_cast<size_t>(kRowsPerCta) * S::template warp_bytes<T>(false);
+  static int per_sm = 0;
+  if (per_sm == 0) per_sm = occupancy(bmr_plan_kernel<T, LOGW, G>, 32 * kRowsPerCta, smem);
+  const int64_t grid = clamp_grid((ap.m + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm);
+  bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p, ap, ncols, pending);
 }
 
 }  // namespace
@@ -220,7 +362,34 @@ void launch_bmr(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStr
   *launches += 1;
 }
 
+template <typename T>
+void launch_bmr_plan(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, int32_t* pending, int num_sms,
+                     cudaStream_t s, int* launches) {
+  // The planning pass uses the smallest register-bitmap bin that covers all columns of B.
+  const int bin = bmr_bin_for_span(ncols);
+#define WS_PLAN(LW)                                                                         \
+  switch (p.log2_group) {                                                                  \
+    case 2: launch_plan_g<T, LW, 4>(p, ap, ncols, pending, num_sms, s); break;             \
+    case 3: launch_plan_g<T, LW, 8>(p, ap, ncols, pending, num_sms, s); break;             \
+    case 4: launch_plan_g<T, LW, 16>(p, ap, ncols, pending, num_sms, s); break;            \
+    default: launch_plan_g<T, LW, 32>(p, ap, ncols, pending, num_sms, s); break;           \
+  }
+  if (bin == 0) {
+    WS_PLAN(bmr_log_words(0))
+  } else if (bin == 1) {
+    WS_PLAN(bmr_log_words(1))
+  } else {
+    WS_PLAN(bmr_log_words(2))
+  }
+#undef WS_PLAN
+  *launches += 1;
+}
+
 template void launch_bmr<float>(const RowPlan<float>&, int, bool, int, cudaStream_t, int*);
 template void launch_bmr<double>(const RowPlan<double>&, int, bool, int, cudaStream_t, int*);
+template void launch_bmr_plan<float>(const RowPlan<float>&, const AnalyzeParams&, int64_t, int32_t*, int,
+                                     cudaStream_t, int*);
+template void launch_bmr_plan<double>(const RowPlan<double>&, const AnalyzeParams&, int64_t, int32_t*, int,
+                                      cudaStream_t, int*);
 
 }  // namespace wsk

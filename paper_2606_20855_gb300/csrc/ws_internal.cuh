@@ -52,7 +52,12 @@ __host__ __device__ constexpr int bitmap_cap(int b) {
 constexpr int kNumBmrBins = 3;
 constexpr int kBmrMaxA = 16;
 constexpr int kBmrCap = 512;  // >= kBmrMaxA * 32 products
+constexpr int kBmrSlots = 512;  // rank slots per register bitmap row (one per possible product)
 __host__ __device__ constexpr int bmr_log_words(int b) { return b == 0 ? 6 : b == 1 ? 9 : 11; }
+// Smallest register bitmap bin whose bitmap covers `span` columns (span <= kMaxBitmapSpan).
+__host__ __device__ constexpr int bmr_bin_for_span(long long span) {
+  return span <= (32ll << bmr_log_words(0)) ? 0 : span <= (32ll << bmr_log_words(1)) ? 1 : 2;
+}
 
 // Row class codes stored per row (uint8).
 constexpr uint8_t kClsEmpty = 0;
@@ -62,6 +67,7 @@ constexpr uint8_t kClsBitmap0 = kClsBmr0 + kNumBmrBins;    // .. + kNumBitmapBin
 constexpr uint8_t kClsHash0 = kClsBitmap0 + kNumBitmapBins;  // .. + kNumHashBins - 1
 constexpr uint8_t kClsDense = kClsHash0 + kNumHashBins;
 constexpr uint8_t kClsSort = kClsDense + 1;
+constexpr uint8_t kClsBmrWide = kClsSort + 1;  // register bitmap rows counted by the planning pass
 
 // Segments of the row permutation: direct rows, register bitmap bins, bitmap
 // bins, hash bins, dense-window rows.
@@ -70,7 +76,8 @@ constexpr int kSegBmr0 = 1;
 constexpr int kSegBitmap0 = kSegBmr0 + kNumBmrBins;
 constexpr int kSegHash0 = kSegBitmap0 + kNumBitmapBins;
 constexpr int kSegDense = kSegHash0 + kNumHashBins;
-constexpr int kNumSegs = kSegDense + 1;
+constexpr int kSegBmrWide = kSegDense + 1;
+constexpr int kNumSegs = kSegBmrWide + 1;
 
 // Device error flags (OR-ed into DevSummary::status).
 enum DevError : int {
@@ -92,7 +99,7 @@ struct DevSummary {
   int n_long;
   int n_empty;
   int bad_row;
-  int pad0;
+  int n_pending;  // rows the planning pass left to the analysis kernel
   int seg_count[kNumSegs];
   int seg_cursor[kNumSegs];
 };
@@ -122,6 +129,7 @@ struct RowPlan {
   const int32_t* slice_idx;
   const int32_t* slice_first;
   int32_t* slice_cnt;          // entries per dense-window slice
+  uint16_t* ranks;             // register bitmap rows: output position of every product, kBmrSlots per row
   DevSummary* sum;
   int64_t seg_begin;   // first position in perm of the segment a kernel processes
   int64_t seg_len;     // rows in that segment
@@ -140,9 +148,13 @@ struct AnalyzeParams {
   int dense_width;
   int long_threshold;
 };
+// rows == nullptr: every row of A; otherwise the first sum->n_pending entries of rows.
 template <typename T>
-void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, int num_sms,
-                    cudaStream_t s, int* launches);
+void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, const int32_t* rows,
+                    int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_bmr_plan(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, int32_t* pending, int num_sms,
+                     cudaStream_t s, int* launches);
 template <typename T>
 void launch_scatter(const RowPlan<T>& p, int64_t m, const int64_t* seg_offset, int num_sms, cudaStream_t s,
                     int* launches);
