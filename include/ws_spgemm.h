@@ -155,8 +155,10 @@ ws_status_t ws_csr_nnz(ws_csr_t handle, int64_t* nnz_out);
  * path, info[4] dense-window rows, info[5] dense-window slices,
  * info[6] total products (sum over rows of the product count),
  * info[7] number of kernel launches queued by the last symbolic pass,
- * info[8] number queued by the last numeric pass, info[9] bitmap rows.
- * `n` is the length of `info` (at most 10 values are written).
+ * info[8] number queued by the last numeric pass, info[9] bitmap rows,
+ * info[10] heavy rows on the dense column-slice path, info[11] heavy rows
+ * on the wide-bitmap path.
+ * `n` is the length of `info` (at most 12 values are written).
  */
 ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
 
@@ -173,6 +175,10 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
  *          (default and maximum 65536; 0 disables the bitmap path)
  *   key 5: most stored A entries of a row that uses the one-warp register
  *          bitmap path (default and maximum 16; 0 disables that path)
+ *   key 6: most stored A entries of a heavy row that uses the dense
+ *          column-slice path (default and maximum 8192; 0 disables it)
+ *   key 7: widest column range of a heavy row that uses the wide-bitmap path
+ *          (default and maximum 1048576; 0 disables it)
  * Returns WS_ERR_INVALID_ARG for an unknown key or out-of-range value.
  */
 ws_status_t ws_set_tuning(int key, int64_t value);

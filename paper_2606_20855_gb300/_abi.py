@@ -124,7 +124,7 @@ def ws_csr_nnz(h: int) -> int:
 
 
 PLAN_INFO_KEYS = ("empty_rows", "direct_rows", "hash_rows", "sorted_rows", "dense_rows", "dense_slices",
-                  "products", "symbolic_launches", "numeric_launches", "bitmap_rows")
+                  "products", "symbolic_launches", "numeric_launches", "bitmap_rows", "rcd_rows", "wb_rows")
 
 
 def ws_spgemm_plan_info(C: int) -> dict:
@@ -133,9 +133,10 @@ def ws_spgemm_plan_info(C: int) -> dict:
     return dict(zip(PLAN_INFO_KEYS, list(arr)))
 
 
-TUNING_KEYS = {"hash_max_products": 1, "run_limit": 2, "dense_width": 3, "bitmap_span": 4, "register_rows_max_a": 5}
+TUNING_KEYS = {"hash_max_products": 1, "run_limit": 2, "dense_width": 3, "bitmap_span": 4, "register_rows_max_a": 5,
+               "dense_rows_max_a": 6, "wide_bitmap_span": 7}
 TUNING_DEFAULTS = {"hash_max_products": 4096, "run_limit": 64, "dense_width": 0, "bitmap_span": 65536,
-                   "register_rows_max_a": 16}
+                   "register_rows_max_a": 16, "dense_rows_max_a": 8192, "wide_bitmap_span": 1 << 20}
 
 
 def ws_set_tuning(key, value: int) -> None:

@@ -26,32 +26,41 @@ __device__ __forceinline__ int ceil_log2_ll(long long x) {  // x >= 1
 // Class of a row from its stored-entry count, product count and column range.
 // Bitmap bins take rows whose range fits a bitmap that is not much larger
 // than the row's products (at most 8 words per product plus 64).
-// Rows with at most kBmrMaxA entries whose B rows fit one lane group take the
-// register bitmap bins.
+// Rows with at most bmr_max_a entries whose B rows fit one lane group take the
+// register bitmap bins; other narrow rows with at most 1024 entries the
+// bitmap bins.  Heavy rows (more entries than those) go to the dense rows
+// (narrow range, few stored A entries: long B rows), the 8192-entry bitmap
+// bin, the hash bins, the wide bitmap (range up to 2^20) and finally the
+// column-sliced dense window.
 __device__ __forceinline__ uint8_t classify(long long nnza, long long ub, int lo, int hi, int maxlen,
                                             const AnalyzeParams& ap) {
   if (ub == 0) return kClsEmpty;
   if (nnza == 1) return kClsDirect;
   const long long span = static_cast<long long>(hi) - lo + 1;
-  if (span <= ap.bitmap_span && ((span + 31) >> 5) <= 8 * ub + 64) {
+  const long long est = ub < span ? ub : span;  // entries of the row are at most this
+  const bool bitmap_ok = span <= ap.bitmap_span && ((span + 31) >> 5) <= 8 * ub + 64;
+  if (bitmap_ok) {
     if (nnza <= ap.bmr_max_a && maxlen <= ap.group) {
 #pragma unroll
       for (int b = 0; b < kNumBmrBins; ++b) {
         if (span <= (32ll << bmr_log_words(b))) return static_cast<uint8_t>(kClsBmr0 + b);
       }
     }
-    const long long est = ub < span ? ub : span;  // entries of the row are at most this
 #pragma unroll
-    for (int b = 0; b < kNumBitmapBins; ++b) {
-      if (span <= (32ll << bitmap_log_words(b)) && est <= bitmap_cap(b))
-        return static_cast<uint8_t>(kClsBitmap0 + b);
+    for (int b = 0; b < kNumBitmapBins - 1; ++b) {
+      if (span <= (32ll << bitmap_log_words(b)) && est <= bitmap_cap(b)) return static_cast<uint8_t>(kClsBitmap0 + b);
     }
   }
+  const bool heavy = ub > 4096 || (bitmap_ok && est > bitmap_cap(kNumBitmapBins - 2));
+  if (heavy && span <= kMaxBitmapSpan && nnza <= ap.rcd_max_a) return kClsRcd;
+  if (bitmap_ok && span <= (32ll << bitmap_log_words(kNumBitmapBins - 1)) && est <= bitmap_cap(kNumBitmapBins - 1))
+    return static_cast<uint8_t>(kClsBitmap0 + kNumBitmapBins - 1);
   if (ub <= ap.hash_max) {
     int b = ceil_log2_ll(ub) - (kMinHashLog - 1);
     b = b < 0 ? 0 : b;
     return static_cast<uint8_t>(kClsHash0 + b);
   }
+  if (span <= ap.wb_span) return kClsWb;
   return kClsDense;
 }
 
@@ -59,6 +68,8 @@ __device__ __forceinline__ int segment_of(uint8_t cls) {
   if (cls == kClsDirect) return kSegDirect;
   if (cls == kClsDense) return kSegDense;
   if (cls == kClsBmrWide) return kSegBmrWide;
+  if (cls == kClsRcd) return kSegRcd;
+  if (cls == kClsWb) return kSegWb;
   if (cls < kClsBitmap0) return kSegBmr0 + (cls - kClsBmr0);      // register bitmap bins
   if (cls < kClsHash0) return kSegBitmap0 + (cls - kClsBitmap0);  // bitmap bins
   return kSegHash0 + (cls - kClsHash0);                            // hash bins
@@ -167,6 +178,7 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
     const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
     long long ub = 0;
     int lo = INT_MAX, hi = -1;
+#pragma unroll 4
     for (int64_t q = s + lane; q < e; q += 32) {
       const int k = p.A.colidx[q];
       const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];

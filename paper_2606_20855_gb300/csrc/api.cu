@@ -29,6 +29,8 @@ thread_local std::string g_last_error;
 int64_t g_hash_max = kMaxHashProducts;
 int64_t g_bitmap_span = kMaxBitmapSpan;
 int g_bmr_max_a = kBmrMaxA;
+int g_rcd_max_a = kRcdDefaultMaxA;
+int64_t g_wb_span = kWbMaxSpan;
 int g_run_limit = 64;
 int g_dense_width = 0;  // 0 = default per value type
 constexpr int kLongRowThreshold = 128;
@@ -249,8 +251,8 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
 
   RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
   if (m > 0) {
-    AnalyzeParams ap{m, g_hash_max, g_bitmap_span, 1 << pl->log2_group, g_bmr_max_a, pl->dense_width,
-                     kLongRowThreshold};
+    AnalyzeParams ap{m,           g_hash_max, g_bitmap_span,   1 << pl->log2_group, g_bmr_max_a,
+                     g_rcd_max_a, g_wb_span,  pl->dense_width, kLongRowThreshold};
     // When every row of C fits the widest register bitmap (B has at most
     // 65,536 columns), the planning pass counts the eligible rows in its first
     // read of A and only the remaining rows go through the analysis kernel.
@@ -300,6 +302,16 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
     p.seg_len = pl->seg_count[kSegDense];
     launch_dense_slices<T>(p, pl->slice_row, pl->slice_idx, pl->slice_first, sms, s, &pl->sym_launches);
     launch_dense<T>(p, pl->dense_slices, false, sms, s, &pl->sym_launches);
+  }
+  if (pl->seg_count[kSegRcd] > 0) {
+    p.seg_begin = pl->seg_offset[kSegRcd];
+    p.seg_len = pl->seg_count[kSegRcd];
+    launch_rcd<T>(p, false, sms, s, &pl->sym_launches);
+  }
+  if (pl->seg_count[kSegWb] > 0) {
+    p.seg_begin = pl->seg_offset[kSegWb];
+    p.seg_len = pl->seg_count[kSegWb];
+    launch_wb<T>(p, false, sms, s, &pl->sym_launches);
   }
   for (int b = 0; b < kNumBmrBins; ++b) {
     const int g = kSegBmr0 + b;
@@ -353,6 +365,16 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     p.seg_begin = pl->seg_offset[kSegBmrWide];
     p.seg_len = pl->seg_count[kSegBmrWide];
     launch_bmr<T>(p, pl->wide_bin, true, sms, s, &pl->num_launches);
+  }
+  if (pl->seg_count[kSegRcd] > 0) {
+    p.seg_begin = pl->seg_offset[kSegRcd];
+    p.seg_len = pl->seg_count[kSegRcd];
+    launch_rcd<T>(p, true, sms, s, &pl->num_launches);
+  }
+  if (pl->seg_count[kSegWb] > 0) {
+    p.seg_begin = pl->seg_offset[kSegWb];
+    p.seg_len = pl->seg_count[kSegWb];
+    launch_wb<T>(p, true, sms, s, &pl->num_launches);
   }
   for (int b = 0; b < kNumBmrBins; ++b) {
     const int g = kSegBmr0 + b;
@@ -552,7 +574,7 @@ ws_status_t ws_csr_nnz(ws_csr_t h, int64_t* nnz_out) {
 ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
   if (!C || !info || n < 0) return fail(WS_ERR_INVALID_ARG, "NULL argument");
   const Plan* pl = C->plan;
-  int64_t v[10] = {0, 0, 0, 0, 0, 0, 0, 0, 0, 0};
+  int64_t v[12] = {0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0};
   if (pl) {
     int64_t hash_rows = 0, bitmap_rows = 0;
     for (int b = 0; b < kNumHashBins; ++b) hash_rows += pl->seg_count[kSegHash0 + b];
@@ -569,8 +591,10 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n) {
     v[7] = pl->sym_launches;
     v[8] = pl->num_launches;
     v[9] = bitmap_rows;
+    v[10] = pl->seg_count[kSegRcd];
+    v[11] = pl->seg_count[kSegWb];
   }
-  for (int i = 0; i < n && i < 10; ++i) info[i] = v[i];
+  for (int i = 0; i < n && i < 12; ++i) info[i] = v[i];
   return WS_OK;
 }
 
@@ -596,6 +620,14 @@ ws_status_t ws_set_tuning(int key, int64_t value) {
     case 5:
       if (value < 0 || value > kBmrMaxA) return fail(WS_ERR_INVALID_ARG, "register-row entry limit out of range");
       g_bmr_max_a = static_cast<int>(value);
+      return WS_OK;
+    case 6:
+      if (value < 0 || value > kRcdMaxA) return fail(WS_ERR_INVALID_ARG, "dense-row entry limit out of range");
+      g_rcd_max_a = static_cast<int>(value);
+      return WS_OK;
+    case 7:
+      if (value < 0 || value > kWbMaxSpan) return fail(WS_ERR_INVALID_ARG, "wide-bitmap span out of range");
+      g_wb_span = value;
       return WS_OK;
   }
   return fail(WS_ERR_INVALID_ARG, "unknown tuning key %d", key);

@@ -10,11 +10,11 @@
 // nnz of the row, and the rank of a column is its position in the sorted
 // output row) and stores, for every product, the rank of its column in the
 // plan (uint16, kBmrSlots slots per row).
-// Numeric pass.  No workspace search is left: every product adds its value
-// at its stored rank in a compact staging array (a shared-memory atomic, the
-// atomic level of Sec. 4, for the rare repeated column), the column goes to
-// the same slot, and the warp copies the sorted row to C with coalesced
-// stores.  One warp owns the row (shard pattern, Sec. 4).
+// Numeric pass.  No workspace search is left: the first product of every
+// column stores its column and value at its stored rank in a compact staging
+// array, the products that repeat a column then add theirs (a shared-memory
+// atomic, the atomic level of Sec. 4), and the warp copies the sorted row to
+// C with coalesced stores.  One warp owns the row (shard pattern, Sec. 4).
 //
 // Lanes are split into groups of G lanes; the group of lane l takes stored A
 // entries j = l / G, l / G + 32/G, ...; lane l takes element l % G of B[k_j,:].
@@ -47,11 +47,12 @@ struct BmrShape {
   static constexpr int kWPL = kWords >= 32 ? kWords / 32 : 1;  // words per lane
   static constexpr int kLogWPL = LOGW >= 5 ? LOGW - 5 : 0;
   static constexpr int kPhysWords = kWPL * 32;
-  // symbolic: bitmap + per-word rank prefix + per-lane base; numeric: staging
+  static constexpr int kSPL = kWPL >= 32 ? kWPL / 32 : 1;  // summary words per lane
+  // symbolic: bitmap + per-word rank prefix + per-lane base + summary; numeric: staging
   template <typename T>
   static constexpr size_t warp_bytes(bool numeric) {
     return numeric ? static_cast<size_t>(kBmrCap) * (4 + sizeof(T))
-                   : static_cast<size_t>(kPhysWords) * 6 + 32 * 4;
+                   : static_cast<size_t>(kPhysWords) * 6 + 32 * 4 + static_cast<size_t>(kSPL) * 32 * 4;
   }
 };
 
@@ -122,18 +123,39 @@ __device__ __forceinline__ void clear_bits(uint32_t* bm, const int* col, int lo)
 }
 
 // Ranks the row's bitmap and stores the rank of every product column at
-// ranks[s * 32 + lane]; clears the words it set; returns nnz of the row.
+// ranks[s * 32 + lane], with bit 15 set when another product of the row
+// already claimed that column (so exactly one product per column has it
+// clear); clears the words it set; returns nnz of the row.
+// A summary bitmap (one bit per bitmap word, lane l's summary words at
+// h * 32 + l) lets each lane visit only the non-zero words it owns.
 template <class S, int kSteps>
-__device__ __forceinline__ int rank_products(uint32_t* bm, uint16_t* pre, int* base, const int* col, int lo, int lane,
-                                             uint16_t* ranks) {
-  set_bits<S, false, kSteps>(bm, col, lo);
+__device__ __forceinline__ int rank_products(uint32_t* bm, uint32_t* sm, uint16_t* pre, int* base, const int* col,
+                                             int lo, int lane, uint16_t* ranks) {
+  uint32_t dup = 0;  // bit s: product s found its column's bit already set
+#pragma unroll
+  for (int s = 0; s < kSteps; ++s) {
+    if (col[s] >= 0) {
+      const uint32_t off = static_cast<uint32_t>(col[s] - lo);
+      const uint32_t w = off >> 5;
+      const uint32_t j = w & (S::kWPL - 1);  // word index inside the owner's range
+      const uint32_t bit = 1u << (off & 31u);
+      if (atomicOr(bm + phys_word<S>(w), bit) & bit) dup |= 1u << s;
+      atomicOr(sm + (((j >> 5) << 5) | (w >> S::kLogWPL)), 1u << (j & 31u));
+    }
+  }
   __syncwarp();
   int run = 0;
-#pragma unroll 8
-  for (int j = 0; j < S::kWPL; ++j) {
-    const int ph = (j << 5) | lane;
-    pre[ph] = static_cast<uint16_t>(run);
-    run += __popc(bm[ph]);
+#pragma unroll
+  for (int h = 0; h < S::kSPL; ++h) {
+    uint32_t m = sm[(h << 5) | lane];
+    sm[(h << 5) | lane] = 0u;  // only this lane reads it
+    while (m) {
+      const int b = __ffs(m) - 1;
+      m &= m - 1u;
+      const int ph = (((h << 5) | b) << 5) | lane;
+      pre[ph] = static_cast<uint16_t>(run);
+      run += __popc(bm[ph]);
+    }
   }
   int incl = run;
 #pragma unroll
@@ -151,7 +173,7 @@ __device__ __forceinline__ int rank_products(uint32_t* bm, uint16_t* pre, int* b
       const uint32_t w = off >> 5;
       const uint32_t ph = phys_word<S>(w);
       const int pos = base[w >> S::kLogWPL] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
-      ranks[(s << 5) | lane] = static_cast<uint16_t>(pos);
+      ranks[(s << 5) | lane] = static_cast<uint16_t>(pos | (((dup >> s) & 1u) << 15));
     }
   }
   __syncwarp();
@@ -161,7 +183,7 @@ __device__ __forceinline__ int rank_products(uint32_t* bm, uint16_t* pre, int* b
 }
 
 template <typename T, int LOGW, int G, bool NUMERIC>
-__global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 5 : 6) bmr_rows_kernel(const RowPlan<T> p) {
+__global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? (sizeof(T) == 8 ? 5 : 7) : 6) bmr_rows_kernel(const RowPlan<T> p) {
   using S = BmrShape<LOGW>;
   constexpr int kSteps = kBmrMaxA / (32 / G);
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -172,12 +194,14 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 5 : 6) bmr_rows_ke
   uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
   uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
   int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
+  uint32_t* sm = reinterpret_cast<uint32_t*>(base + 32);
   // numeric workspace
   int* st_key = reinterpret_cast<int*>(ws);
   T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kBmrCap) * 4);
 
   if constexpr (!NUMERIC) {
     for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
+    for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
     __syncwarp();
   }
 
@@ -192,7 +216,7 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 5 : 6) bmr_rows_ke
     load_products<T, G, NUMERIC, kSteps>(p, ra, na, lane, col, val);
 
     if constexpr (!NUMERIC) {
-      const int total = rank_products<S, kSteps>(bm, pre, base, col, p.lo[row], lane, ranks);
+      const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, p.lo[row], lane, ranks);
       if (lane == 0) p.c_rowptr[row + 1] = total;
     } else {
       int rk[kSteps];
@@ -202,22 +226,32 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? 5 : 6) bmr_rows_ke
       const int64_t want = p.c_rowptr[row + 1] - cbase;
       const int cnt = static_cast<int>(want < kBmrCap ? want : kBmrCap);  // staging bounds every access
       if (lane == 0 && want > kBmrCap) atomicOr(&p.sum->status, kErrCount);
-      for (int s2 = lane; s2 < cnt; s2 += 32) st_val[s2] = T(0);
-      __syncwarp();
-      bool bad = false;
+      // The first product of every column stores its value; the rare repeats add theirs after.
+      bool bad = false, repeats = false;
 #pragma unroll
       for (int s = 0; s < kSteps; ++s) {
         if (col[s] >= 0) {
-          if (rk[s] < cnt) {
-            st_key[rk[s]] = col[s];
-            atomicAdd(&st_val[rk[s]], val[s]);
-          } else {
+          const int r = rk[s] & 0x7fff;
+          if (r >= cnt) {
             bad = true;
+          } else if (rk[s] & 0x8000) {
+            repeats = true;
+          } else {
+            st_key[r] = col[s];
+            st_val[r] = val[s];
           }
         }
       }
       if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
       __syncwarp();
+      if (__any_sync(kFull, repeats)) {
+#pragma unroll
+        for (int s = 0; s < kSteps; ++s) {
+          const int r = rk[s] & 0x7fff;
+          if (col[s] >= 0 && (rk[s] & 0x8000) && r < cnt) atomicAdd(&st_val[r], val[s]);
+        }
+        __syncwarp();
+      }
       for (int s2 = lane; s2 < cnt; s2 += 32) {
         p.c_colidx[cbase + s2] = st_key[s2];
         p.c_vals[cbase + s2] = st_val[s2];
@@ -246,11 +280,13 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const Row
   uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
   uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
   int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
+  uint32_t* sm = reinterpret_cast<uint32_t*>(base + 32);
   if (threadIdx.x == 0) {
     s_taken = 0;
     s_prod = 0;
   }
   for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
+  for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
   __syncthreads();
   const long long words = (ncols + 31) >> 5;
   int taken = 0;
@@ -280,7 +316,7 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const Row
         int col[kSteps];
         T unused[kSteps];
         load_products<T, G, false, kSteps>(p, ra, na, lane, col, unused);
-        const int total = rank_products<S, kSteps>(bm, pre, base, col, 0, lane, p.ranks + row * kBmrSlots);
+        const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, 0, lane, p.ranks + row * kBmrSlots);
         if (lane == 0) {
           p.c_rowptr[row + 1] = total;
           p.cls[row] = kClsBmrWide;

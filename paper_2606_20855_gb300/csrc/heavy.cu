@@ -1,0 +1,347 @@
+// Heavy rows: rows with too many products for the one-warp workspaces.  One
+// CTA owns one row (the shard pattern of Sec. 4), so every output segment is
+// written by one CTA and no CTA waits on another.
+//
+// Dense rows (kClsRcd): the row's column range is at most 65,536 columns and
+// it has at most kRcdMaxA stored A entries (typically hub rows: few stored A
+// entries whose B rows are long).  This is the dense workspace of Gustavson's
+// algorithm (Sec. 5.1) -- a value per column plus a flag per column, the
+// sparse byte-map workspace -- over column slices:
+//   symbolic: every product stores 1 into the flag byte of its column (plain
+//             byte stores, no atomics: the store is idempotent); nnz of the
+//             row is the number of set flags.
+//   numeric:  for each slice of `width` columns, groups of lanes walk the B
+//             rows of the stored A entries from their cursors (where the
+//             previous slice stopped) and add a * b into the dense value
+//             window with shared-memory atomics (the atomic level of Sec. 4).
+//             The flags of the slice are then scanned in column order, so the
+//             slice's entries are written sorted.
+//
+// Wide rows (kClsWb): column range up to 2^20 columns.  A bitmap over the
+// whole range (one bit per column) is the workspace:
+//   symbolic: atomicOr every product column, count the bits that were 0.
+//   numeric:  set the bits, rank the bitmap in 128-bit chunks, write C's
+//             column indices in order straight from the bitmap, zero C's
+//             values, and let every product add its value at the rank of its
+//             column in C (global atomic add; the row's segment is private).
+#include <climits>
+
+#include "ws_internal.cuh"
+
+namespace wsk {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kRcdThreads = 256;
+constexpr int kRcdNumThreads = 512;
+constexpr int kWbThreads = 512;
+
+// ---------------------------------------------------------------- dense rows
+
+// Counts the non-zero bytes of 16 bytes.
+__device__ __forceinline__ int nonzero_bytes(const uint4 v) {
+  return __popc(__vcmpne4(v.x, 0u) & 0x01010101u) + __popc(__vcmpne4(v.y, 0u) & 0x01010101u) +
+         __popc(__vcmpne4(v.z, 0u) & 0x01010101u) + __popc(__vcmpne4(v.w, 0u) & 0x01010101u);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowPlan<T> p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint8_t* flags = smem_raw;  // kMaxBitmapSpan bytes
+  uint4* flags4 = reinterpret_cast<uint4*>(smem_raw);
+  __shared__ long long s_scan[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kWarps = kRcdThreads / 32;
+  for (int i = threadIdx.x; i < kMaxBitmapSpan / 16; i += kRcdThreads) flags4[i] = make_uint4(0u, 0u, 0u, 0u);
+  __syncthreads();
+  for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
+    const int32_t row = p.perm[p.seg_begin + r];
+    const int lo = p.lo[row];
+    const int span = p.hi[row] - lo + 1;
+    const int64_t ra = p.A.rowptr[row], re = p.A.rowptr[row + 1];
+    for (int64_t pa = ra + warp; pa < re; pa += kWarps) {
+      const int k = p.A.colidx[pa];
+      const int64_t qe = p.B.rowptr[k + 1];
+      int64_t q = p.B.rowptr[k] + lane;
+      for (; q + 96 < qe; q += 128) {  // four loads in flight per lane
+        const int c0 = p.B.colidx[q], c1 = p.B.colidx[q + 32], c2 = p.B.colidx[q + 64], c3 = p.B.colidx[q + 96];
+        flags[c0 - lo] = 1;
+        flags[c1 - lo] = 1;
+        flags[c2 - lo] = 1;
+        flags[c3 - lo] = 1;
+      }
+      for (; q < qe; q += 32) flags[p.B.colidx[q] - lo] = 1;
+    }
+    __syncthreads();
+    long long cnt = 0;
+    const int n16 = (span + 15) >> 4;
+    for (int i = threadIdx.x; i < n16; i += kRcdThreads) {
+      cnt += nonzero_bytes(flags4[i]);
+      flags4[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    long long total;
+    block_exclusive_scan(cnt, s_scan, &total);
+    if (threadIdx.x == 0) p.c_rowptr[row + 1] = total;
+    __syncthreads();
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const RowPlan<T> p, int width) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  T* dense = reinterpret_cast<T*>(smem_raw);                           // width values
+  uint8_t* flags = smem_raw + static_cast<size_t>(width) * sizeof(T);  // width bytes
+  int* a_cur = reinterpret_cast<int*>(flags + width);                  // kRcdMaxA cursors (offset in B row)
+  __shared__ long long s_scan[32];
+  const int lg = p.log2_group;
+  const int gsize = 1 << lg;
+  const int grp = threadIdx.x >> lg;
+  const int gl = threadIdx.x & (gsize - 1);
+  const int ngrp = kRcdNumThreads >> lg;
+  const unsigned gmask = gsize == 32 ? kFull : (((1u << gsize) - 1u) << ((threadIdx.x & 31) & ~(gsize - 1)));
+  for (int i = threadIdx.x; i < width; i += kRcdNumThreads) {
+    dense[i] = T(0);
+    flags[i] = 0;
+  }
+  __syncthreads();
+  for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
+    const int32_t row = p.perm[p.seg_begin + r];
+    const int lo = p.lo[row];
+    const int hi = p.hi[row];
+    const int64_t ra = p.A.rowptr[row];
+    const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);  // <= kRcdMaxA by classification
+    const int64_t cbase = p.c_rowptr[row];
+    const int64_t cend = p.c_rowptr[row + 1];
+    for (int j = threadIdx.x; j < na; j += kRcdNumThreads) a_cur[j] = 0;
+    __syncthreads();
+    int64_t emitted = 0;
+    bool bad = false;
+    for (long long c0 = lo; c0 <= hi; c0 += width) {
+      const long long c1 = min(c0 + width, static_cast<long long>(hi) + 1);
+      // Every group of lanes walks the B rows of its stored A entries from
+      // their cursors; products of one B row have distinct columns, products
+      // of different groups meet in shared-memory atomics.
+      for (int j = grp; j < na; j += ngrp) {
+        const int k = p.A.colidx[ra + j];
+        const T av = p.A.vals[ra + j];
+        const int64_t b0 = p.B.rowptr[k];
+        const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        int t = a_cur[j] + gl;
+        int stop = len;
+        for (; t < len; t += gsize) {
+          const int c = p.B.colidx[b0 + t];
+          if (c >= c1) {
+            stop = t;
+            break;
+          }
+          const int off = static_cast<int>(c - c0);
+          atomicAdd(dense + off, av * p.B.vals[b0 + t]);
+          flags[off] = 1;
+        }
+        // new cursor: the first position of the B row at or past c1
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          if (o < gsize) stop = min(stop, __shfl_xor_sync(gmask, stop, o));
+        }
+        if (gl == 0) a_cur[j] = stop;
+      }
+      __syncthreads();
+      // Emit the slice in column order.
+      const int w = static_cast<int>(c1 - c0);
+      const int per = (w + kRcdNumThreads - 1) / kRcdNumThreads;  // consecutive columns per thread
+      const int my0 = threadIdx.x * per;
+      const int my1 = min(my0 + per, w);
+      long long mine = 0;
+      for (int i = my0; i < my1; ++i) mine += flags[i] != 0;
+      long long total;
+      const long long ex = block_exclusive_scan(mine, s_scan, &total);
+      int64_t pos = cbase + emitted + ex;
+      for (int i = my0; i < my1; ++i) {
+        if (flags[i]) {
+          if (pos < cend) {
+            p.c_colidx[pos] = static_cast<int32_t>(c0 + i);
+            p.c_vals[pos] = dense[i];
+          } else {
+            bad = true;
+          }
+          ++pos;
+          flags[i] = 0;
+          dense[i] = T(0);
+        }
+      }
+      emitted += total;
+      __syncthreads();
+    }
+    if (threadIdx.x == 0 && emitted != cend - cbase) bad = true;
+    if (bad) atomicOr(&p.sum->status, kErrCount);
+  }
+}
+
+// ----------------------------------------------------------------- wide rows
+
+template <typename T, bool NUMERIC>
+__global__ void __launch_bounds__(kWbThreads, 1) wb_kernel(const RowPlan<T> p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint32_t* bm = reinterpret_cast<uint32_t*>(smem_raw);          // kWbMaxSpan / 32 words
+  uint4* bm4 = reinterpret_cast<uint4*>(smem_raw);
+  uint32_t* pre = bm + kWbMaxSpan / 32;                           // one prefix per 128-bit chunk
+  __shared__ long long s_scan[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kWarps = kWbThreads / 32;
+  const int lg = p.log2_group;
+  const int gsize = 1 << lg;
+  const int grp = threadIdx.x >> lg;
+  const int gl = threadIdx.x & (gsize - 1);
+  const int ngrp = kWbThreads >> lg;
+  (void)warp;
+  (void)kWarps;
+  for (int i = threadIdx.x; i < kWbMaxSpan / 128; i += kWbThreads) bm4[i] = make_uint4(0u, 0u, 0u, 0u);
+  __syncthreads();
+  for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
+    const int32_t row = p.perm[p.seg_begin + r];
+    const int lo = p.lo[row];
+    const int span = p.hi[row] - lo + 1;
+    const int nchunks = (span + 127) >> 7;
+    const int64_t ra = p.A.rowptr[row], re = p.A.rowptr[row + 1];
+    int64_t cbase = 0, cend = 0;
+    if constexpr (NUMERIC) {
+      cbase = p.c_rowptr[row];
+      cend = p.c_rowptr[row + 1];
+      for (int64_t i = cbase + threadIdx.x; i < cend; i += kWbThreads) p.c_vals[i] = T(0);
+    }
+    // Set the bit of every product column.
+    long long fresh = 0;
+    for (int64_t pa = ra + grp; pa < re; pa += ngrp) {
+      const int k = p.A.colidx[pa];
+      const int64_t qe = p.B.rowptr[k + 1];
+      for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
+        const uint32_t off = static_cast<uint32_t>(p.B.colidx[q] - lo);
+        const uint32_t bit = 1u << (off & 31u);
+        if constexpr (NUMERIC) {
+          atomicOr(bm + (off >> 5), bit);
+        } else {
+          fresh += (atomicOr(bm + (off >> 5), bit) & bit) == 0u;
+        }
+      }
+    }
+    __syncthreads();
+    if constexpr (!NUMERIC) {
+      long long total;
+      block_exclusive_scan(fresh, s_scan, &total);
+      if (threadIdx.x == 0) p.c_rowptr[row + 1] = total;
+      for (int i = threadIdx.x; i < nchunks; i += kWbThreads) bm4[i] = make_uint4(0u, 0u, 0u, 0u);
+      __syncthreads();
+    } else {
+      // Rank the chunks: thread t owns a run of consecutive chunks.
+      const int per = (nchunks + kWbThreads - 1) / kWbThreads;
+      const int my0 = threadIdx.x * per;
+      const int my1 = min(my0 + per, nchunks);
+      long long mine = 0;
+      for (int i = my0; i < my1; ++i) {
+        const uint4 v = bm4[i];
+        mine += __popc(v.x) + __popc(v.y) + __popc(v.z) + __popc(v.w);
+      }
+      long long total;
+      long long run = block_exclusive_scan(mine, s_scan, &total);
+      bool bad = total != cend - cbase;
+      // Write the column indices in order and keep each chunk's prefix.
+      for (int i = my0; i < my1; ++i) {
+        pre[i] = static_cast<uint32_t>(run);
+        const uint4 v = bm4[i];
+        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t x = wv[q];
+          while (x) {
+            const int b = __ffs(x) - 1;
+            x &= x - 1u;
+            const int64_t pos = cbase + run;
+            if (pos < cend) p.c_colidx[pos] = lo + (i << 7) + (q << 5) + b;
+            ++run;
+          }
+        }
+      }
+      __syncthreads();  // prefixes and the zeroed values are visible to the CTA
+      for (int64_t pa = ra + grp; pa < re; pa += ngrp) {
+        const int k = p.A.colidx[pa];
+        const T av = p.A.vals[pa];
+        const int64_t qe = p.B.rowptr[k + 1];
+        for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
+          const uint32_t off = static_cast<uint32_t>(p.B.colidx[q] - lo);
+          const uint32_t i = off >> 7;
+          const uint4 v = bm4[i];
+          const uint32_t wq = (off >> 5) & 3u;
+          const uint32_t wd = wq == 0 ? v.x : wq == 1 ? v.y : wq == 2 ? v.z : v.w;
+          const int64_t pos = cbase + pre[i] + (wq > 0 ? __popc(v.x) : 0) + (wq > 1 ? __popc(v.y) : 0) +
+                              (wq > 2 ? __popc(v.z) : 0) + __popc(wd & ((1u << (off & 31u)) - 1u));
+          if (pos < cend) {
+            atomicAdd(p.c_vals + pos, av * p.B.vals[q]);
+          } else {
+            bad = true;
+          }
+        }
+      }
+      if (bad) atomicOr(&p.sum->status, kErrCount);
+      __syncthreads();
+      for (int i = threadIdx.x; i < nchunks; i += kWbThreads) bm4[i] = make_uint4(0u, 0u, 0u, 0u);
+      __syncthreads();
+    }
+  }
+}
+
+template <typename K>
+int occupancy(K kern, int threads, size_t smem) {
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  int n = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, smem);
+  return n > 0 ? n : 1;
+}
+
+int grid_of(int64_t rows, int num_sms, int per_sm) {
+  int64_t g = rows;
+  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
+  if (g > cap) g = cap;
+  if (g < 1) g = 1;
+  return static_cast<int>(g);
+}
+
+}  // namespace
+
+size_t rcd_numeric_smem(int width, size_t value_bytes) {
+  return static_cast<size_t>(width) * (value_bytes + 1) + static_cast<size_t>(kRcdMaxA) * 4;
+}
+
+template <typename T>
+void launch_rcd(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches) {
+  if (!numeric) {
+    const size_t smem = kMaxBitmapSpan;
+    static int per_sm = 0;
+    if (per_sm == 0) per_sm = occupancy(rcd_symbolic_kernel<T>, kRcdThreads, smem);
+    rcd_symbolic_kernel<T><<<grid_of(p.seg_len, num_sms, per_sm), kRcdThreads, smem, s>>>(p);
+  } else {
+    const int width = kRcdWidthBytes / static_cast<int>(sizeof(T));
+    const size_t smem = rcd_numeric_smem(width, sizeof(T));
+    static int per_sm = 0;
+    if (per_sm == 0) per_sm = occupancy(rcd_numeric_kernel<T>, kRcdNumThreads, smem);
+    rcd_numeric_kernel<T><<<grid_of(p.seg_len, num_sms, per_sm), kRcdNumThreads, smem, s>>>(p, width);
+  }
+  *launches += 1;
+}
+
+template <typename T>
+void launch_wb(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches) {
+  const size_t smem = kWbMaxSpan / 8 + (kWbMaxSpan / 128) * 4;
+  auto kern = numeric ? wb_kernel<T, true> : wb_kernel<T, false>;
+  static int per_sm[2] = {0, 0};
+  if (per_sm[numeric] == 0) per_sm[numeric] = occupancy(kern, kWbThreads, smem);
+  kern<<<grid_of(p.seg_len, num_sms, per_sm[numeric]), kWbThreads, smem, s>>>(p);
+  *launches += 1;
+}
+
+template void launch_rcd<float>(const RowPlan<float>&, bool, int, cudaStream_t, int*);
+template void launch_rcd<double>(const RowPlan<double>&, bool, int, cudaStream_t, int*);
+template void launch_wb<float>(const RowPlan<float>&, bool, int, cudaStream_t, int*);
+template void launch_wb<double>(const RowPlan<double>&, bool, int, cudaStream_t, int*);
+
+}  // namespace wsk

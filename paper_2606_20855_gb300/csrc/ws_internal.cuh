@@ -68,6 +68,14 @@ constexpr uint8_t kClsHash0 = kClsBitmap0 + kNumBitmapBins;  // .. + kNumHashBin
 constexpr uint8_t kClsDense = kClsHash0 + kNumHashBins;
 constexpr uint8_t kClsSort = kClsDense + 1;
 constexpr uint8_t kClsBmrWide = kClsSort + 1;  // register bitmap rows counted by the planning pass
+constexpr uint8_t kClsRcd = kClsBmrWide + 1;    // heavy rows, dense column-slice workspace, CTA per row
+constexpr uint8_t kClsWb = kClsRcd + 1;         // heavy rows, wide bitmap workspace, CTA per row
+
+// Heavy-row limits.
+constexpr int kRcdMaxA = 8192;            // stored A entries a dense row may have (cursor slots)
+constexpr int kRcdDefaultMaxA = 8192;     // default limit used by the classification
+constexpr int kRcdWidthBytes = 65536;     // dense value window per slice
+constexpr int kWbMaxSpan = 1 << 20;       // widest column range of a wide-bitmap row
 
 // Segments of the row permutation: direct rows, register bitmap bins, bitmap
 // bins, hash bins, dense-window rows.
@@ -77,7 +85,9 @@ constexpr int kSegBitmap0 = kSegBmr0 + kNumBmrBins;
 constexpr int kSegHash0 = kSegBitmap0 + kNumBitmapBins;
 constexpr int kSegDense = kSegHash0 + kNumHashBins;
 constexpr int kSegBmrWide = kSegDense + 1;
-constexpr int kNumSegs = kSegBmrWide + 1;
+constexpr int kSegRcd = kSegBmrWide + 1;
+constexpr int kSegWb = kSegRcd + 1;
+constexpr int kNumSegs = kSegWb + 1;
 
 // Device error flags (OR-ed into DevSummary::status).
 enum DevError : int {
@@ -145,6 +155,8 @@ struct AnalyzeParams {
   int64_t bitmap_span; // largest column range that uses a bitmap bin (0: none)
   int group;           // lanes per stored A entry in the register bitmap kernels
   int bmr_max_a;       // most stored A entries of a register bitmap row (0: none)
+  int rcd_max_a;       // most stored A entries of a dense heavy row (0: no dense heavy rows)
+  int64_t wb_span;     // widest column range of a wide-bitmap heavy row (0: none)
   int dense_width;
   int long_threshold;
 };
@@ -167,6 +179,10 @@ template <typename T>
 void launch_bmr(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_bitmap(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_rcd(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_wb(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_dense(const RowPlan<T>& p, int64_t nslices, bool numeric, int num_sms, cudaStream_t s,
                   int* launches);

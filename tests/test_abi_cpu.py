@@ -76,7 +76,7 @@ def test_host_argument_errors(lib):
 
 def test_tuning_knob_validation(lib):
     try:
-        for key, bad in [(1, -1), (1, 5000), (2, 0), (3, 1000), (3, 20480), (4, -1), (4, 65537), (5, 17), (9, 1)]:
+        for key, bad in [(1, -1), (1, 5000), (2, 0), (3, 1000), (3, 20480), (4, -1), (4, 65537), (5, 17), (6, 8193), (7, (1 << 20) + 1), (9, 1)]:
             with pytest.raises(_abi.WsError):
                 _abi.ws_set_tuning(key, bad)
         _abi.ws_set_tuning("hash_max_products", 0)

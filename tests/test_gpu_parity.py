@@ -91,7 +91,8 @@ def test_every_row_class(dtype, n):
     A = _csr(len(lens) * 3, k, rows, dtype=dtype)
     A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
     rowptr, colidx, vals, info = run_gpu(A, B, validate=True)
-    assert info["direct_rows"] == 6 and info["empty_rows"] == 3 and info["dense_rows"] > 0
+    assert info["direct_rows"] == 6 and info["empty_rows"] == 3
+    assert info["dense_rows"] + info["rcd_rows"] + info["wb_rows"] > 0
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
@@ -100,7 +101,7 @@ def test_dense_window_path_everywhere(dtype):
     rng = np.random.default_rng(12)
     A = uniform_csr(3000, 800, 6, rng, dtype, "sym")
     B = uniform_csr(800, 9000, 12, rng, dtype, "sym")
-    with tuning(hash_max_products=0, dense_width=1024, bitmap_span=0):
+    with tuning(hash_max_products=0, dense_width=1024, bitmap_span=0, wide_bitmap_span=0):
         rowptr, colidx, vals, info = run_gpu(A, B)
     assert info["hash_rows"] == 0 and info["dense_rows"] == 3000 and info["dense_slices"] > 3000
     assert_matches_oracle(A, B, rowptr, colidx, vals)
@@ -117,6 +118,51 @@ def test_sort_path_everywhere(dtype):
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
+HEAVY = {"default": {}, "no_dense_rows": {"dense_rows_max_a": 0}, "wide_bitmap_only": {"dense_rows_max_a": 0, "bitmap_span": 0},
+         "sliced_only": {"dense_rows_max_a": 0, "bitmap_span": 0, "wide_bitmap_span": 0, "hash_max_products": 0},
+         "dense_rows_few_a": {"dense_rows_max_a": 64}}
+
+
+@pytest.mark.parametrize("heavy", list(HEAVY))
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_heavy_rows(heavy, dtype):
+    """Hub rows of a skewed product (few stored A entries, long B rows) and
+    wide rows with many short B rows, on every heavy-row path."""
+    rng = np.random.default_rng(31)
+    rp, ci, _ = rmat_pattern(13, 16, (0.57, 0.19, 0.19, 0.05), rng)
+    A = HostCSR(8192, 8192, rp, ci, (1.0 - rng.random(ci.size)).astype(dtype))
+    from synth import row_subset
+    from tests._helpers import products_per_row
+    lens, ub = np.diff(rp), products_per_row(A, A)
+    hubs = np.argsort(lens)[-100:]                               # many stored entries
+    fed = np.flatnonzero((ub > 4096) & (lens <= 64))[:300]      # few entries, long (hub) B rows
+    light = rng.choice(8192, size=100, replace=False)
+    H = row_subset(A, np.unique(np.concatenate([hubs, fed, light])))
+    with tuning(**HEAVY[heavy]):
+        rowptr, colidx, vals, info = run_gpu(H, A)
+    if heavy == "default":
+        assert info["rcd_rows"] > 0
+    if heavy == "wide_bitmap_only":
+        assert info["wb_rows"] > 0
+    if heavy == "sliced_only":
+        assert info["dense_rows"] > 0
+    assert_matches_oracle(H, A, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_wide_heavy_rows(dtype):
+    """Rows with thousands of stored A entries over short B rows spanning ~2^20 columns."""
+    rng = np.random.default_rng(32)
+    k, n = 20_000, 1 << 20
+    B = uniform_csr(k, n, 4, rng, dtype, "pos")
+    rows = {i: rng.choice(k, size=int(L), replace=False).tolist() for i, L in enumerate([1500, 3000, 6000, 2, 40])}
+    A = _csr(5, k, rows, dtype=dtype)
+    A.vals = (1.0 - rng.random(A.nnz)).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["wb_rows"] == 3
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
 @pytest.mark.parametrize("path", list(PATHS))
 def test_skewed_rmat_square(path):
     rng = np.random.default_rng(14)
@@ -125,7 +171,7 @@ def test_skewed_rmat_square(path):
     with tuning(**PATHS[path]):
         rowptr, colidx, vals, info = run_gpu(A, A)
     if path == "hash":
-        assert info["dense_rows"] > 0 and info["bitmap_rows"] == 0
+        assert info["dense_rows"] + info["rcd_rows"] + info["wb_rows"] > 0 and info["bitmap_rows"] == 0
     else:
         assert info["bitmap_rows"] > 0
     assert_matches_oracle(A, A, rowptr, colidx, vals)
@@ -173,7 +219,7 @@ def test_single_dense_row_and_wide_output():
     A.vals = 2 * rng.random(A.nnz) - 1
     B = uniform_csr(k, n, 30, rng)
     rowptr, colidx, vals, info = run_gpu(A, B)
-    assert info["dense_rows"] == 1
+    assert info["wb_rows"] == 1
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
