@@ -94,12 +94,8 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
   uint8_t* flags = smem_raw + static_cast<size_t>(width) * sizeof(T);  // width bytes
   int* a_cur = reinterpret_cast<int*>(flags + width);                  // kRcdMaxA cursors (offset in B row)
   __shared__ long long s_scan[32];
-  const int lg = p.log2_group;
-  const int gsize = 1 << lg;
-  const int grp = threadIdx.x >> lg;
-  const int gl = threadIdx.x & (gsize - 1);
-  const int ngrp = kRcdNumThreads >> lg;
-  const unsigned gmask = gsize == 32 ? kFull : (((1u << gsize) - 1u) << ((threadIdx.x & 31) & ~(gsize - 1)));
+  constexpr int kWarps = kRcdNumThreads / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int i = threadIdx.x; i < width; i += kRcdNumThreads) {
     dense[i] = T(0);
     flags[i] = 0;
@@ -119,56 +115,73 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
     bool bad = false;
     for (long long c0 = lo; c0 <= hi; c0 += width) {
       const long long c1 = min(c0 + width, static_cast<long long>(hi) + 1);
-      // Every group of lanes walks the B rows of its stored A entries from
-      // their cursors; products of one B row have distinct columns, products
-      // of different groups meet in shared-memory atomics.
-      for (int j = grp; j < na; j += ngrp) {
+      // Every warp walks the B rows of its stored A entries from their cursors,
+      // four loads in flight per lane; the columns of one B row are distinct,
+      // entries of different warps meet in shared-memory atomics.
+      for (int j = warp; j < na; j += kWarps) {
         const int k = p.A.colidx[ra + j];
         const T av = p.A.vals[ra + j];
         const int64_t b0 = p.B.rowptr[k];
         const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
-        int t = a_cur[j] + gl;
         int stop = len;
-        for (; t < len; t += gsize) {
-          const int c = p.B.colidx[b0 + t];
-          if (c >= c1) {
-            stop = t;
-            break;
-          }
-          const int off = static_cast<int>(c - c0);
-          atomicAdd(dense + off, av * p.B.vals[b0 + t]);
-          flags[off] = 1;
-        }
-        // new cursor: the first position of the B row at or past c1
+        for (int t0 = a_cur[j]; t0 < len; t0 += 128) {
+          int cc[4];
+          T bv[4];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          if (o < gsize) stop = min(stop, __shfl_xor_sync(gmask, stop, o));
+          for (int u = 0; u < 4; ++u) {
+            const int t = t0 + u * 32 + lane;
+            cc[u] = t < len ? p.B.colidx[b0 + t] : INT_MAX;
+            bv[u] = t < len ? p.B.vals[b0 + t] : T(0);
+          }
+          bool past = false;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int t = t0 + u * 32 + lane;
+            if (cc[u] < c1) {
+              const int off = static_cast<int>(cc[u] - c0);
+              atomicAdd(dense + off, av * bv[u]);
+              flags[off] = 1;
+            } else if (t < len) {
+              stop = min(stop, t);
+              past = true;
+            }
+          }
+          if (__any_sync(kFull, past)) break;  // the rest of this B row lies past the slice
         }
-        if (gl == 0) a_cur[j] = stop;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) stop = min(stop, __shfl_xor_sync(kFull, stop, o));
+        if (lane == 0) a_cur[j] = stop;
       }
       __syncthreads();
-      // Emit the slice in column order.
+      // Emit the slice in column order: warp w owns a contiguous block of
+      // columns, read 32 at a time (ballot compaction, coalesced stores).
       const int w = static_cast<int>(c1 - c0);
-      const int per = (w + kRcdNumThreads - 1) / kRcdNumThreads;  // consecutive columns per thread
-      const int my0 = threadIdx.x * per;
-      const int my1 = min(my0 + per, w);
+      const int per_warp = ((w + kWarps * 32 - 1) / (kWarps * 32)) * 32;
+      const int wb0 = warp * per_warp;
+      const int wb1 = min(wb0 + per_warp, w);
       long long mine = 0;
-      for (int i = my0; i < my1; ++i) mine += flags[i] != 0;
+      for (int i = wb0 + lane; i < wb1; i += 32) mine += flags[i] != 0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mine += __shfl_xor_sync(kFull, mine, o);
       long long total;
-      const long long ex = block_exclusive_scan(mine, s_scan, &total);
-      int64_t pos = cbase + emitted + ex;
-      for (int i = my0; i < my1; ++i) {
-        if (flags[i]) {
-          if (pos < cend) {
-            p.c_colidx[pos] = static_cast<int32_t>(c0 + i);
-            p.c_vals[pos] = dense[i];
+      const long long ex = block_exclusive_scan(lane == 0 ? mine : 0ll, s_scan, &total);
+      int64_t pos = cbase + emitted + __shfl_sync(kFull, ex, 0);
+      for (int i0 = wb0; i0 < wb1; i0 += 32) {
+        const int i = i0 + lane;
+        const bool f = i < wb1 && flags[i] != 0;
+        const unsigned m = __ballot_sync(kFull, f);
+        if (f) {
+          const int64_t q = pos + __popc(m & ((1u << lane) - 1u));
+          if (q < cend) {
+            p.c_colidx[q] = static_cast<int32_t>(c0 + i);
+            p.c_vals[q] = dense[i];
           } else {
             bad = true;
           }
-          ++pos;
           flags[i] = 0;
           dense[i] = T(0);
         }
+        pos += __popc(m);
       }
       emitted += total;
       __syncthreads();
