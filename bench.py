@@ -43,6 +43,11 @@ METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per con
 DEFAULT_WORKLOAD = "uniform_rect_1m"
 NOMINAL_HBM_GBS = 8000.0
 
+# DRAM bytes (read + write) of one numeric-pass launch at full size, from the ncu
+# capture summarised in profiles/bmr_kernels_uniform_rect_1m_262144rows.md
+# (262,144-row case scaled by rows).  Valid only for the kernels it was taken on.
+NUMERIC_TRAFFIC = {"uniform_rect_1m": 5.68e9}
+
 
 def products_per_row(A, B) -> np.ndarray:
     lenB = np.diff(B.rowptr)
@@ -66,37 +71,44 @@ def measured_peaks() -> dict:
 
 
 class ClockSampler:
-    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+    """Samples SM clocks and throttle reasons with nvidia-smi while running.
 
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    Samples carry nvidia-smi's own timestamps; `stop(t0, t1)` keeps those taken
+    inside the wall-clock window [t0, t1] (widened to 0.5 s around it when the
+    window is shorter than the sampling period)."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index: int):
+    def __init__(self, index: int, period_ms: int = 25):
         self.index = index
+        self.period_ms = period_ms
         self.proc = None
-        self.lines: list[str] = []
+        self.lines: list[tuple[float, str]] = []
         self._t = None
 
     def start(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", str(self.period_ms)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except (OSError, ValueError):
             self.proc = None
             return self
         self._t = threading.Thread(target=self._read, daemon=True)
         self._t.start()
+        time.sleep(0.3)  # let the first samples arrive before the timed region
         return self
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
 
-    def stop(self) -> dict | None:
+    def stop(self, t0: float, t1: float) -> dict | None:
         if not self.proc:
             return None
+        time.sleep(0.1)
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
@@ -104,24 +116,45 @@ class ClockSampler:
             self.proc.kill()
         if self._t:
             self._t.join(timeout=2)
-        sm, smax, reasons = [], [], set()
+        pad = 0.0 if (t1 - t0) > 4 * self.period_ms / 1e3 else 0.5
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
-            parts = [p.strip() for p in ln.split(",")]
-            if len(parts) < 8:
+        sm, smax, reasons = [], [], set()
+        for when, ln in self.lines:
+            if not (t0 - pad <= when <= t1 + pad):
+                continue
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
                 continue
             try:
-                sm.append(float(parts[0]))
-                smax.append(float(parts[1]))
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
             except ValueError:
                 continue
-            for nm, val in zip(names, parts[4:8]):
+            for nm, val in zip(names, parts[5:9]):
                 if val.lower() == "active":
                     reasons.add(nm)
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "window_s": round(t1 - t0, 3)}
+
+
+def oracle_sample(A, B, target_s: float, rng, cores: int) -> tuple[np.ndarray, float]:
+    """A seeded uniform row sample on which the oracle runs for about target_s
+    seconds (grown from 1024 rows by 4x until a run takes a quarter of the
+    target, then scaled), and the time of its last sizing run."""
+    from oracle import oracle_spgemm
+    n = min(A.nrows, 1024)
+    while True:
+        rows = np.sort(rng.choice(A.nrows, size=n, replace=False))
+        t0 = time.perf_counter()
+        oracle_spgemm(A, B, rows=rows, threads=cores)
+        dt = time.perf_counter() - t0
+        if dt >= 0.25 * target_s or n >= A.nrows:
+            break
+        n = min(A.nrows, n * 4)
+    want = int(n * target_s / max(dt, 1e-6))
+    return np.sort(rng.choice(A.nrows, size=min(A.nrows, max(n, want)), replace=False)), dt
 
 
 def cpu_baseline(A, B, ub: np.ndarray, target_s: float, seed: int = 0) -> dict:
@@ -129,14 +162,8 @@ def cpu_baseline(A, B, ub: np.ndarray, target_s: float, seed: int = 0) -> dict:
     from oracle import oracle_spgemm
     cores = os.cpu_count() or 1
     rng = np.random.default_rng(seed)
-    probe = np.sort(rng.choice(A.nrows, size=min(A.nrows, 512), replace=False))
-    t0 = time.perf_counter()
-    oracle_spgemm(A, B, rows=probe, threads=cores)
-    dt = max(time.perf_counter() - t0, 1e-6)
-    per_product = dt / max(int(ub[probe].sum()), 1)
-    want_products = target_s / per_product
-    nrows = int(min(A.nrows, max(probe.size, want_products / max(ub.mean(), 1e-9))))
-    rows = np.sort(rng.choice(A.nrows, size=nrows, replace=False))
+    rows, _ = oracle_sample(A, B, target_s, rng, cores)
+    nrows = rows.size
     t0 = time.perf_counter()
     oracle_spgemm(A, B, rows=rows, threads=cores)
     dt = time.perf_counter() - t0
@@ -144,6 +171,17 @@ def cpu_baseline(A, B, ub: np.ndarray, target_s: float, seed: int = 0) -> dict:
     return {"value": round(2.0 * prods / dt / 1e9, 4), "unit": "GFLOP/s", "cores": cores, "kind": "oracle",
             "sample": f"{nrows} of {A.nrows} rows (seeded uniform sample, {prods} products), "
                       f"{dt:.1f} s, std::map per row, {cores} threads"}
+
+
+def numeric_kernels(info: dict) -> str:
+    """Which numeric kernels a plan launches (from ws_spgemm_plan_info)."""
+    names = []
+    for key, kern in (("direct_rows", "direct_rows_kernel"), ("bitmap_rows", "bmr_rows/bitmap_rows_kernel"),
+                      ("hash_rows", "hash_rows_kernel"), ("sorted_rows", "sort_rows_kernel"),
+                      ("rcd_rows", "rcd_numeric_kernel"), ("wb_rows", "wb_kernel"), ("dense_rows", "dense_rows_kernel")):
+        if info.get(key):
+            names.append(kern)
+    return ", ".join(names) or "none"
 
 
 def dist_setup():
@@ -194,13 +232,8 @@ def run_reference(args, world, rank) -> None:
     ub = products_per_row(A, B)
     cores = os.cpu_count() or 1
     rng = np.random.default_rng(1234)
-    # size one step to about args.ref_step_s seconds
-    probe = np.sort(rng.choice(A.nrows, size=min(A.nrows, 512), replace=False))
-    t0 = time.perf_counter()
-    oracle_spgemm(A, B, rows=probe, threads=cores)
-    per_product = max(time.perf_counter() - t0, 1e-6) / max(int(ub[probe].sum()), 1)
-    nrows = int(min(A.nrows, max(probe.size, args.ref_step_s / per_product / max(ub.mean(), 1e-9))))
-    rows = np.sort(rng.choice(A.nrows, size=nrows, replace=False))
+    rows, _ = oracle_sample(A, B, args.ref_step_s, rng, cores)  # one step ~ ref_step_s seconds
+    nrows = rows.size
     prods = int(ub[rows].sum())
     for _ in range(args.warmup):
         oracle_spgemm(A, B, rows=rows, threads=cores)
@@ -263,6 +296,7 @@ def run_ours(args, world, rank, local, pg) -> None:
     clocks = ClockSampler(local).start() if rank == 0 else None
     barrier(world, pg)
     torch.cuda.synchronize(device)
+    t_wall0 = time.time()
     for i in range(args.steps):
         flush.fill_(i)  # write > L2 between timed steps (not timed)
         e0, e1, e2 = ev[i]
@@ -273,8 +307,9 @@ def run_ours(args, world, rank, local, pg) -> None:
         e2.record(stream)
         op.wait()
     torch.cuda.synchronize(device)
+    t_wall1 = time.time()
     barrier(world, pg)
-    clk = clocks.stop() if clocks else None
+    clk = clocks.stop(t_wall0, t_wall1) if clocks else None
     step_ms = [a.elapsed_time(c) for a, _, c in ev]
     num_ms = [b.elapsed_time(c) for _, b, c in ev]
     sym_ms = [a.elapsed_time(b) for a, b, _ in ev]
@@ -351,9 +386,11 @@ def run_ours(args, world, rank, local, pg) -> None:
                       "numeric_median": round(statistics.median(num_ms), 4),
                       "step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
         "roofline": {
-            "kernel": "numeric pass (hash-bin rows)", "bound": "hbm", "achieved": round(num_achieved, 1),
+            "kernel": f"numeric pass ({info['numeric_launches']} launch(es): {numeric_kernels(info)})",
+            "bound": "hbm", "achieved": round(num_achieved, 1),
             "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(num_achieved / peaks["hbm_gbs"], 4),
-            "peak_source": peaks["source"], "traffic": args.traffic,
+            "peak_source": peaks["source"], "algorithmic_bytes": int(algo_bytes),
+            "traffic": args.traffic if args.traffic is not None else (None if args.rows else NUMERIC_TRAFFIC.get(args.workload)),
         },
         "gpu_launches": int(launches_per_step * args.steps),
         "plan": info,
@@ -367,13 +404,13 @@ def run_ours(args, world, rank, local, pg) -> None:
 def main(argv=None) -> int:
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=list(WORKLOADS), default=DEFAULT_WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
-    ap.add_argument("--ref-step-s", type=float, default=4.0, help="seconds per reference-arm step")
+    ap.add_argument("--ref-step-s", type=float, default=2.0, help="seconds per reference-arm step")
     ap.add_argument("--rows", type=int, default=0,
                     help="use only the first ROWS rows of A (a smaller case of the same workload, for profiling)")
     ap.add_argument("--traffic", type=float, default=None,
