@@ -183,6 +183,30 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
  */
 ws_status_t ws_set_tuning(int key, int64_t value);
 
+/*
+ * ws_rowptr_scan_static -- builds a CSR row pointer from per-row counts
+ * without allocating any memory.  (The paper has no counterpart: this is a
+ * service for callers of this library that cannot allocate device memory at
+ * this point, for example code inside a framework that owns all device
+ * memory and forbids outside allocations, or a latency-critical loop where
+ * cudaMalloc/cudaFree would block on the whole device.)
+ *   rowptr  device int64[nrows + 1]; on entry rowptr[i + 1] holds the entry
+ *           count of row i (rowptr[0] is ignored); on exit rowptr[0] = 0 and
+ *           rowptr[i + 1] = rowptr[i] + count_i, so rowptr[nrows] = nnz.
+ *   nrows   0 <= nrows <= 16,777,216 (the fixed scratch holds one partial
+ *           sum per 4096 rows); larger values return WS_ERR_OVERFLOW.
+ *   stream  the work is queued on it; the call does not wait.
+ * Scratch lives in a fixed array compiled into the library (about 33 KB),
+ * which every GPU that loads the library keeps until the process exits.  The
+ * call itself calls no cudaMalloc, cudaFree or other allocating routine.
+ * The first call on a device looks up that array's device address; make
+ * that first call before any stream capture.  All calls share the array:
+ * calls that may run at the same time on the GPU (on unordered streams) race
+ * and give wrong results.  Returns WS_ERR_INVALID_ARG for a NULL rowptr or a
+ * negative nrows, WS_ERR_CUDA if a CUDA call fails.
+ */
+ws_status_t ws_rowptr_scan_static(int64_t* rowptr, int64_t nrows, ws_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

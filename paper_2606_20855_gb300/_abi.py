@@ -42,6 +42,7 @@ SIGNATURES = [
     ("ws_csr_nnz", _i32, [_p, ctypes.POINTER(_i64)]),
     ("ws_spgemm_plan_info", _i32, [_p, ctypes.POINTER(_i64), _i32]),
     ("ws_set_tuning", _i32, [_i32, _i64]),
+    ("ws_rowptr_scan_static", _i32, [_p, _i64, _p]),
 ]
 
 
@@ -142,3 +143,11 @@ TUNING_DEFAULTS = {"hash_max_products": 4096, "run_limit": 64, "dense_width": 0,
 def ws_set_tuning(key, value: int) -> None:
     k = TUNING_KEYS[key] if isinstance(key, str) else int(key)
     _check("ws_set_tuning", load().ws_set_tuning(k, int(value)))
+
+
+def ws_rowptr_scan_static(rowptr: int, nrows: int, stream: int) -> None:
+    """Allocation-free row-pointer scan (see include/ws_spgemm.h): rowptr[1:]
+    holds per-row counts on entry and the prefix sums on exit."""
+    status = load().ws_rowptr_scan_static(rowptr or None, nrows, stream or None)
+    if status != 0:
+        raise WsError("ws_rowptr_scan_static", status, STATUS_NAMES.get(status, str(status)))

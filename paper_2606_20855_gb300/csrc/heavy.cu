@@ -200,15 +200,11 @@ __global__ void __launch_bounds__(kWbThreads, 1) wb_kernel(const RowPlan<T> p) {
   uint4* bm4 = reinterpret_cast<uint4*>(smem_raw);
   uint32_t* pre = bm + kWbMaxSpan / 32;                           // one prefix per 128-bit chunk
   __shared__ long long s_scan[32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  constexpr int kWarps = kWbThreads / 32;
   const int lg = p.log2_group;
   const int gsize = 1 << lg;
   const int grp = threadIdx.x >> lg;
   const int gl = threadIdx.x & (gsize - 1);
   const int ngrp = kWbThreads >> lg;
-  (void)warp;
-  (void)kWarps;
   for (int i = threadIdx.x; i < kWbMaxSpan / 128; i += kWbThreads) bm4[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncthreads();
   for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
