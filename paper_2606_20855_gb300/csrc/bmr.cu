@@ -26,10 +26,10 @@
 // step, and the 32 sorted columns of one B row mostly fall in different
 // banks.  After use, a row clears only the words it set.
 //
-// Planning.  When B has at most 65,536 columns every row fits the widest
-// bitmap with lo = 0, and bmr_plan_kernel handles every eligible row of A in
-// the first pass over A (no separate analysis pass for those rows); the rows
-// it does not take are queued for the analysis kernel.
+// Planning.  When B has at most 65,536 columns every row fits a bitmap over
+// all columns (lo = 0), and bmr_plan_kernel ranks every eligible row of A in
+// the first pass over A, two warps per row (no separate analysis pass for
+// those rows); the rows it does not take are queued for the analysis kernel.
 #include <climits>
 
 #include "ws_internal.cuh"
@@ -266,44 +266,73 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? (sizeof(T) == 8 ? 
 // and a bitmap of at most 8 words per product is ranked right here (class
 // kClsBmrWide, lo = 0); every other row goes to `pending` for the analysis
 // kernel.  Counts per class are added to the summary.
-template <typename T, int LOGW, int G>
-__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
-                                                                   int64_t ncols, int32_t* pending) {
-  using S = BmrShape<LOGW>;
-  constexpr int kSteps = kBmrMaxA / (32 / G);
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ int s_taken;
-  __shared__ unsigned long long s_prod;
-  const int sub = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::template warp_bytes<T>(false);
-  uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
-  uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
-  int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
-  uint32_t* sm = reinterpret_cast<uint32_t*>(base + 32);
-  if (threadIdx.x == 0) {
-    s_taken = 0;
-    s_prod = 0;
+//
+// One CTA of kPlanThreads threads (two warps) works on one row, so the
+// bitmap of a row is shared by all of them: thread t owns the contiguous
+// words [t * WPT, (t + 1) * WPT), stored at (w % WPT) * kPlanThreads + w / WPT.  Product
+// (stored A entry j, element e of B[k_j,:]) keeps the slot j * G + e, the
+// same slot the one-warp numeric kernel uses.
+#ifndef WS_PLAN_THREADS
+#define WS_PLAN_THREADS 64
+#endif
+constexpr int kPlanThreads = WS_PLAN_THREADS;
+
+template <int LOGW>
+struct PlanShape {
+  static constexpr int kWords = 1 << LOGW;
+  static constexpr int kWPT = kWords >= kPlanThreads ? kWords / kPlanThreads : 1;  // words per thread
+  static constexpr int kLogThreads = kPlanThreads == 64 ? 6 : kPlanThreads == 128 ? 7 : 8;
+  static constexpr int kLogWPT = LOGW >= kLogThreads ? LOGW - kLogThreads : 0;
+  static constexpr int kPhysWords = kWPT * kPlanThreads;
+  static constexpr int kSPT = kWPT >= 32 ? kWPT / 32 : 1;  // summary words per thread
+  static constexpr size_t bytes() {
+    return static_cast<size_t>(kPhysWords) * 6 + kPlanThreads * 4 + static_cast<size_t>(kSPT) * kPlanThreads * 4;
   }
-  for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
-  for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
+};
+
+template <class S>
+__device__ __forceinline__ uint32_t plan_phys(uint32_t w) {
+  return (w & (S::kWPT - 1)) * kPlanThreads + (w >> S::kLogWPT);
+}
+
+template <typename T, int LOGW, int G>
+__global__ void __launch_bounds__(kPlanThreads, 1024 / kPlanThreads) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
+                                                                int64_t ncols, int32_t* pending) {
+  using S = PlanShape<LOGW>;
+  constexpr int kGroups = kPlanThreads / G;   // A entries per step
+  constexpr int kSteps = (kBmrMaxA + kGroups - 1) / kGroups;  // steps covering kBmrMaxA entries
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint32_t* bm = reinterpret_cast<uint32_t*>(smem_raw);
+  uint16_t* pre = reinterpret_cast<uint16_t*>(smem_raw + static_cast<size_t>(S::kPhysWords) * 4);
+  int* base = reinterpret_cast<int*>(smem_raw + static_cast<size_t>(S::kPhysWords) * 6);
+  uint32_t* sm = reinterpret_cast<uint32_t*>(base + kPlanThreads);
+  __shared__ long long s_b0[kBmrMaxA];
+  __shared__ int s_len[kBmrMaxA];
+  __shared__ int s_red[2 * (kPlanThreads / 32)];
+  __shared__ long long s_scan[32];
+  const int t = threadIdx.x;
+  const int lane = t & 31, warp = t >> 5;
+  const int grp = t / G, gl = t % G;
+  for (int i = t; i < S::kPhysWords; i += kPlanThreads) bm[i] = 0u;
+  for (int i = t; i < S::kSPT * kPlanThreads; i += kPlanThreads) sm[i] = 0u;
   __syncthreads();
   const long long words = (ncols + 31) >> 5;
   int taken = 0;
   unsigned long long prod = 0;
 
-  for (int64_t row = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub; row < ap.m;
-       row += static_cast<int64_t>(gridDim.x) * kRowsPerCta) {
+  for (int64_t row = blockIdx.x; row < ap.m; row += gridDim.x) {
     const int64_t ra = p.A.rowptr[row];
     const int64_t na64 = p.A.rowptr[row + 1] - ra;
     bool ok = na64 >= 2 && na64 <= ap.bmr_max_a;
     const int na = static_cast<int>(ok ? na64 : 0);
     if (ok) {
-      // lane j < na: length of B row k_j
       int my_len = 0;
-      if (lane < na) {
-        const int k = p.A.colidx[ra + lane];
-        my_len = static_cast<int>(p.B.rowptr[k + 1] - p.B.rowptr[k]);
+      if (t < na) {
+        const int k = p.A.colidx[ra + t];
+        const long long b0 = p.B.rowptr[k];
+        my_len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        s_b0[t] = b0;
+        s_len[t] = my_len;
       }
       int ub = my_len, mx = my_len;
 #pragma unroll
@@ -311,13 +340,76 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const Row
         ub += __shfl_xor_sync(kFull, ub, o);
         mx = max(mx, __shfl_xor_sync(kFull, mx, o));
       }
+      constexpr int kW = kPlanThreads / 32;
+      if (lane == 0) {
+        s_red[warp] = ub;
+        s_red[kW + warp] = mx;
+      }
+      __syncthreads();
+      ub = 0;
+      mx = 0;
+#pragma unroll
+      for (int w2 = 0; w2 < kW; ++w2) {
+        ub += s_red[w2];
+        mx = max(mx, s_red[kW + w2]);
+      }
       ok = ub > 0 && mx <= G && words <= 8ll * ub + 64;
       if (ok) {
+        // products of this thread: step s covers A entry j = s * kGroups + grp
         int col[kSteps];
-        T unused[kSteps];
-        load_products<T, G, false, kSteps>(p, ra, na, lane, col, unused);
-        const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, 0, lane, p.ranks + row * kBmrSlots);
-        if (lane == 0) {
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          const int j = st * kGroups + grp;
+          col[st] = -1;
+          if (j < na && gl < s_len[j]) col[st] = p.B.colidx[s_b0[j] + gl];
+        }
+        uint32_t dup = 0;
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          if (col[st] >= 0) {
+            const uint32_t off = static_cast<uint32_t>(col[st]);
+            const uint32_t w = off >> 5;
+            const uint32_t jw = w & (S::kWPT - 1);
+            const uint32_t bit = 1u << (off & 31u);
+            if (atomicOr(bm + plan_phys<S>(w), bit) & bit) dup |= 1u << st;
+            atomicOr(sm + (jw >> 5) * kPlanThreads + (w >> S::kLogWPT), 1u << (jw & 31u));
+          }
+        }
+        __syncthreads();
+        int run = 0;
+#pragma unroll
+        for (int h = 0; h < S::kSPT; ++h) {
+          uint32_t m = sm[h * kPlanThreads + t];
+          sm[h * kPlanThreads + t] = 0u;  // only this thread reads it
+          while (m) {
+            const int b = __ffs(m) - 1;
+            m &= m - 1u;
+            const int ph = ((h << 5) | b) * kPlanThreads + t;
+            pre[ph] = static_cast<uint16_t>(run);
+            run += __popc(bm[ph]);
+          }
+        }
+        long long total;
+        base[t] = static_cast<int>(block_exclusive_scan(static_cast<long long>(run), s_scan, &total));
+        __syncthreads();
+        uint16_t* ranks = p.ranks + row * kBmrSlots;
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          if (col[st] >= 0) {
+            const uint32_t off = static_cast<uint32_t>(col[st]);
+            const uint32_t w = off >> 5;
+            const uint32_t ph = plan_phys<S>(w);
+            const int pos = base[w >> S::kLogWPT] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
+            const int j = st * kGroups + grp;
+            ranks[j * G + gl] = static_cast<uint16_t>(pos | (((dup >> st) & 1u) << 15));
+          }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          if (col[st] >= 0) bm[plan_phys<S>(static_cast<uint32_t>(col[st]) >> 5)] = 0u;
+        }
+        if (t == 0) {
           p.c_rowptr[row + 1] = total;
           p.cls[row] = kClsBmrWide;
           p.lo[row] = 0;
@@ -326,17 +418,13 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_plan_kernel(const Row
           prod += static_cast<unsigned long long>(ub);
         }
       }
+      __syncthreads();  // bitmap clear and s_b0/s_len reuse
     }
-    if (!ok && lane == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
+    if (!ok && t == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
   }
-  if (lane == 0) {
-    atomicAdd(&s_taken, taken);
-    atomicAdd(&s_prod, prod);
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    if (s_taken) atomicAdd(&p.sum->seg_count[kSegBmrWide], s_taken);
-    if (s_prod) atomicAdd(reinterpret_cast<unsigned long long*>(&p.sum->products), s_prod);
+  if (t == 0) {
+    if (taken) atomicAdd(&p.sum->seg_count[kSegBmrWide], taken);
+    if (prod) atomicAdd(reinterpret_cast<unsigned long long*>(&p.sum->products), prod);
   }
 }
 
@@ -377,12 +465,11 @@ void launch_bmr_w(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s
 template <typename T, int LOGW, int G>
 void launch_plan_g(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, int32_t* pending, int num_sms,
                    cudaStream_t s) {
-  using S = BmrShape<LOGW>;
-  const size_t smem = static_cast<size_t>(kRowsPerCta) * S::template warp_bytes<T>(false);
+  const size_t smem = PlanShape<LOGW>::bytes();
   static int per_sm = 0;
-  if (per_sm == 0) per_sm = occupancy(bmr_plan_kernel<T, LOGW, G>, 32 * kRowsPerCta, smem);
-  const int64_t grid = clamp_grid((ap.m + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm);
-  bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p, ap, ncols, pending);
+  if (per_sm == 0) per_sm = occupancy(bmr_plan_kernel<T, LOGW, G>, kPlanThreads, smem);
+  const int64_t grid = clamp_grid(ap.m, num_sms, per_sm);
+  bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), kPlanThreads, smem, s>>>(p, ap, ncols, pending);
 }
 
 }  // namespace
