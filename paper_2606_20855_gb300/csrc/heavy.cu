@@ -154,21 +154,31 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
       }
       __syncthreads();
       // Emit the slice in column order: warp w owns a contiguous block of
-      // columns, read 32 at a time (ballot compaction, coalesced stores).
+      // 32-column chunks (at most 32), finds the touched ones with one 32-byte
+      // flag read per lane, and compacts them with ballots (coalesced stores).
       const int w = static_cast<int>(c1 - c0);
-      const int per_warp = ((w + kWarps * 32 - 1) / (kWarps * 32)) * 32;
-      const int wb0 = warp * per_warp;
-      const int wb1 = min(wb0 + per_warp, w);
+      const int nchunks = (w + 31) >> 5;
+      const int per_warp = (nchunks + kWarps - 1) / kWarps;
+      const int ch0 = warp * per_warp;
+      const int ch1 = min(ch0 + per_warp, nchunks);
+      bool touched = false;
+      if (ch0 + lane < ch1) {
+        const uint4* f4 = reinterpret_cast<const uint4*>(flags + ((ch0 + lane) << 5));
+        const uint4 x = f4[0], y = f4[1];
+        touched = (x.x | x.y | x.z | x.w | y.x | y.y | y.z | y.w) != 0u;
+      }
+      const unsigned tmask = __ballot_sync(kFull, touched);
       long long mine = 0;
-      for (int i = wb0 + lane; i < wb1; i += 32) mine += flags[i] != 0;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) mine += __shfl_xor_sync(kFull, mine, o);
+      for (unsigned tm = tmask; tm; tm &= tm - 1u) {
+        const int i = ((ch0 + __ffs(tm) - 1) << 5) + lane;
+        mine += __popc(__ballot_sync(kFull, i < w && flags[i] != 0));
+      }
       long long total;
       const long long ex = block_exclusive_scan(lane == 0 ? mine : 0ll, s_scan, &total);
       int64_t pos = cbase + emitted + __shfl_sync(kFull, ex, 0);
-      for (int i0 = wb0; i0 < wb1; i0 += 32) {
-        const int i = i0 + lane;
-        const bool f = i < wb1 && flags[i] != 0;
+      for (unsigned tm = tmask; tm; tm &= tm - 1u) {
+        const int i = ((ch0 + __ffs(tm) - 1) << 5) + lane;
+        const bool f = i < w && flags[i] != 0;
         const unsigned m = __ballot_sync(kFull, f);
         if (f) {
           const int64_t q = pos + __popc(m & ((1u << lane) - 1u));
