@@ -12,8 +12,9 @@ C once, at their stored widths).
 
 Extra keys: `e2e` (the same product through the public Python API from
 pinned host inputs to the host copy of C, copies inside the timed region),
-`roofline` (the numeric pass, the dominant launch, against the measured
-copy bandwidth), `cpu_baseline` (the CPU oracle on a bounded row sample, on
+`roofline` (the whole product -- symbolic + numeric, the span the throughput
+target is set on -- against the measured copy bandwidth, with each pass's own
+figure under `passes`), `cpu_baseline` (the CPU oracle on a bounded row sample, on
 this host's cores), `clocks` (nvidia-smi samples during the timed region).
 
 Under torchrun (N > 1) every rank runs its own replica of the workload on its
@@ -43,10 +44,14 @@ METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per con
 DEFAULT_WORKLOAD = "uniform_rect_1m"
 NOMINAL_HBM_GBS = 8000.0
 
-# DRAM bytes (read + write) of one numeric-pass launch at full size, from the ncu
-# capture summarised in profiles/bmr_kernels_uniform_rect_1m_262144rows.md
-# (262,144-row case scaled by rows).  Valid only for the kernels it was taken on.
-NUMERIC_TRAFFIC = {"uniform_rect_1m": 5.68e9}
+# DRAM bytes (read + write) per pass at full size, from the ncu capture
+# summarised in profiles/bmr_kernels_uniform_rect_1m_262144rows.md: the
+# 262,144-row cut scaled by 4 to 1,048,576 rows (both passes stream their
+# rows, so traffic grows in proportion).  Symbolic: bmr_plan_kernel only (the
+# analysis, scatter and scan kernels move a few MB).  Valid only for the
+# kernels they were taken on.
+NUMERIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.415403e9 + 1.019798e9)}
+SYMBOLIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.027999e9 + 0.218566e9)}
 
 
 def products_per_row(A, B) -> np.ndarray:
@@ -173,10 +178,18 @@ def cpu_baseline(A, B, ub: np.ndarray, target_s: float, seed: int = 0) -> dict:
                       f"{dt:.1f} s, std::map per row, {cores} threads"}
 
 
+def roofline_obj(nbytes: int, seconds: float, peaks: dict, traffic) -> dict:
+    """Compulsory bytes over the measured mean duration, against the measured copy bandwidth."""
+    achieved = nbytes / seconds / 1e9
+    return {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": round(achieved / peaks["hbm_gbs"], 4), "peak_source": peaks["source"],
+            "algorithmic_bytes": int(nbytes), "mean_ms": round(seconds * 1e3, 4), "traffic": traffic}
+
+
 def numeric_kernels(info: dict) -> str:
     """Which numeric kernels a plan launches (from ws_spgemm_plan_info)."""
     names = []
-    for key, kern in (("direct_rows", "direct_rows_kernel"), ("bitmap_rows", "bmr_rows/bitmap_rows_kernel"),
+    for key, kern in (("direct_rows", "direct_rows_kernel"), ("bitmap_rows", "bmr_numeric/bitmap_rows_kernel"),
                       ("hash_rows", "hash_rows_kernel"), ("sorted_rows", "sort_rows_kernel"),
                       ("rcd_rows", "rcd_numeric_kernel"), ("wb_rows", "wb_kernel"), ("dense_rows", "dense_rows_kernel")):
         if info.get(key):
@@ -290,6 +303,8 @@ def run_ours(args, world, rank, local, pg) -> None:
     nnz = op.nnz
     info = op.plan_info()
     algo_bytes = csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz, s)
+    # symbolic pass: read the structure of A and B once, write C.rowptr
+    sym_bytes = csr_bytes(A.nrows, A.nnz, 0) + csr_bytes(B.nrows, B.nnz, 0) + 8 * (A.nrows + 1)
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
@@ -354,7 +369,17 @@ def run_ours(args, world, rank, local, pg) -> None:
         return
     peaks = measured_peaks()
     num_mean_s = statistics.mean(num_ms) / 1e3
-    num_achieved = algo_bytes / num_mean_s / 1e9
+
+    def traffic(table):
+        """ncu DRAM bytes for this workload (None: not captured on these kernels, or a row cut)."""
+        if args.rows:
+            return None
+        if table is None:  # whole product: both passes, when both were captured
+            sym, num = traffic(SYMBOLIC_TRAFFIC), traffic(NUMERIC_TRAFFIC)
+            return None if sym is None or num is None else sym + num
+        if table is NUMERIC_TRAFFIC and args.traffic is not None:
+            return args.traffic
+        return table.get(args.workload)
     value = 2.0 * products * args.steps * world / total_s / 1e9
     eff_gbs = algo_bytes * args.steps * world / total_s / 1e9
     base = None
@@ -385,13 +410,16 @@ def run_ours(args, world, rank, local, pg) -> None:
         "phases_ms": {"symbolic_median": round(statistics.median(sym_ms), 4),
                       "numeric_median": round(statistics.median(num_ms), 4),
                       "step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
-        "roofline": {
-            "kernel": f"numeric pass ({info['numeric_launches']} launch(es): {numeric_kernels(info)})",
-            "bound": "hbm", "achieved": round(num_achieved, 1),
-            "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(num_achieved / peaks["hbm_gbs"], 4),
-            "peak_source": peaks["source"], "algorithmic_bytes": int(algo_bytes),
-            "traffic": args.traffic if args.traffic is not None else (None if args.rows else NUMERIC_TRAFFIC.get(args.workload)),
-        },
+        "roofline": dict(roofline_obj(algo_bytes, statistics.mean(step_ms) / 1e3, peaks, traffic(None)),
+                         kernel="whole product: symbolic pass (nnz read-back included) + numeric pass",
+                         passes={
+                             "symbolic": dict(roofline_obj(sym_bytes, statistics.mean(sym_ms) / 1e3, peaks,
+                                                           traffic(SYMBOLIC_TRAFFIC)),
+                                              kernel="symbolic pass (compulsory bytes: structure of A and B "
+                                                     "read once, C.rowptr written)"),
+                             "numeric": dict(roofline_obj(algo_bytes, num_mean_s, peaks, traffic(NUMERIC_TRAFFIC)),
+                                             kernel=f"numeric pass: {numeric_kernels(info)}"),
+                         }),
         "gpu_launches": int(launches_per_step * args.steps),
         "plan": info,
         "clocks": clk,

@@ -18,7 +18,7 @@
 //
 // Lanes are split into groups of G lanes; the group of lane l takes stored A
 // entries j = l / G, l / G + 32/G, ...; lane l takes element l % G of B[k_j,:].
-// Product (step s, lane l) has slot s * 32 + l.
+// The ranks of a lane's steps s and s + steps/2 share one 32-bit slot.
 //
 // Bitmap layout.  With WPL = words / 32 words per lane, word w is stored at
 // (w % WPL) * 32 + w / WPL: lane l owns the contiguous words [l*WPL, (l+1)*WPL)
@@ -30,6 +30,7 @@
 // all columns (lo = 0), and bmr_plan_kernel ranks every eligible row of A in
 // the first pass over A, two warps per row (no separate analysis pass for
 // those rows); the rows it does not take are queued for the analysis kernel.
+// Its numeric pass is bmr_numeric_kernel, as for the binned rows.
 #include <climits>
 
 #include "ws_internal.cuh"
@@ -48,17 +49,27 @@ struct BmrShape {
   static constexpr int kLogWPL = LOGW >= 5 ? LOGW - 5 : 0;
   static constexpr int kPhysWords = kWPL * 32;
   static constexpr int kSPL = kWPL >= 32 ? kWPL / 32 : 1;  // summary words per lane
-  // symbolic: bitmap + per-word rank prefix + per-lane base + summary; numeric: staging
-  template <typename T>
-  static constexpr size_t warp_bytes(bool numeric) {
-    return numeric ? static_cast<size_t>(kBmrCap) * (4 + sizeof(T))
-                   : static_cast<size_t>(kPhysWords) * 6 + 32 * 4 + static_cast<size_t>(kSPL) * 32 * 4;
+  // bitmap + per-word rank prefix + per-lane base + summary
+  static constexpr size_t bytes() {
+    return static_cast<size_t>(kPhysWords) * 6 + 32 * 4 + static_cast<size_t>(kSPL) * 32 * 4;
   }
 };
 
 template <class S>
 __device__ __forceinline__ uint32_t phys_word(uint32_t w) {
   return ((w & (S::kWPL - 1)) << 5) | (w >> S::kLogWPL);
+}
+
+// Rank slots.  In the one-warp kernels lane `lane` holds, at step st of
+// kSteps, the product of stored A entry st * (32 / G) + lane / G.  Steps q and
+// q + kSteps / 2 of a lane (A entries j and j + 8) share the 32-bit word
+// (q * 32 + lane): low half step q, high half step q + kSteps / 2, so the
+// numeric pass fetches two ranks per load and the symbolic passes write whole
+// words.
+template <int kSteps>
+__device__ __forceinline__ int rank_word(int st, int lane) { return ((st % (kSteps / 2)) << 5) | lane; }
+__device__ __forceinline__ uint32_t rank_pack(int lo_rank, int hi_rank) {
+  return static_cast<uint32_t>(lo_rank & 0xffff) | (static_cast<uint32_t>(hi_rank & 0xffff) << 16);
 }
 
 // Loads the row's products into registers: lane j < na first loads stored A
@@ -123,7 +134,7 @@ __device__ __forceinline__ void clear_bits(uint32_t* bm, const int* col, int lo)
 }
 
 // Ranks the row's bitmap and stores the rank of every product column at
-// ranks[s * 32 + lane], with bit 15 set when another product of the row
+// its rank slot, with bit 15 set when another product of the row
 // already claimed that column (so exactly one product per column has it
 // clear); clears the words it set; returns nnz of the row.
 // A summary bitmap (one bit per bitmap word, lane l's summary words at
@@ -166,15 +177,22 @@ __device__ __forceinline__ int rank_products(uint32_t* bm, uint32_t* sm, uint16_
   base[lane] = incl - run;
   const int total = __shfl_sync(kFull, incl, 31);
   __syncwarp();
+  int rk[kSteps];
 #pragma unroll
   for (int s = 0; s < kSteps; ++s) {
+    rk[s] = 0;
     if (col[s] >= 0) {
       const uint32_t off = static_cast<uint32_t>(col[s] - lo);
       const uint32_t w = off >> 5;
       const uint32_t ph = phys_word<S>(w);
       const int pos = base[w >> S::kLogWPL] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
-      ranks[(s << 5) | lane] = static_cast<uint16_t>(pos | (((dup >> s) & 1u) << 15));
+      rk[s] = pos | static_cast<int>(((dup >> s) & 1u) << 15);
     }
+  }
+  uint32_t* ranks32 = reinterpret_cast<uint32_t*>(ranks);
+#pragma unroll
+  for (int q = 0; q < kSteps / 2; ++q) {
+    if (col[q] >= 0 || col[q + kSteps / 2] >= 0) ranks32[rank_word<kSteps>(q, lane)] = rank_pack(rk[q], rk[q + kSteps / 2]);
   }
   __syncwarp();
   clear_bits<S, kSteps>(bm, col, lo);
@@ -182,63 +200,154 @@ __device__ __forceinline__ int rank_products(uint32_t* bm, uint32_t* sm, uint16_
   return total;
 }
 
-template <typename T, int LOGW, int G, bool NUMERIC>
-__global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? (sizeof(T) == 8 ? 5 : 7) : 6) bmr_rows_kernel(const RowPlan<T> p) {
+template <typename T, int LOGW, int G>
+__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const RowPlan<T> p) {
   using S = BmrShape<LOGW>;
   constexpr int kSteps = kBmrMaxA / (32 / G);
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::template warp_bytes<T>(NUMERIC);
-  // symbolic workspace
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::bytes();
   uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
   uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
   int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
   uint32_t* sm = reinterpret_cast<uint32_t*>(base + 32);
-  // numeric workspace
-  int* st_key = reinterpret_cast<int*>(ws);
-  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kBmrCap) * 4);
-
-  if constexpr (!NUMERIC) {
-    for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
-    for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
-    __syncwarp();
-  }
+  for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
+  for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
+  __syncwarp();
 
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub; r < p.seg_len;
        r += static_cast<int64_t>(gridDim.x) * kRowsPerCta) {
     const int32_t row = p.perm[p.seg_begin + r];
     const int64_t ra = p.A.rowptr[row];
     const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
-    uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
     int col[kSteps];
     T val[kSteps];
-    load_products<T, G, NUMERIC, kSteps>(p, ra, na, lane, col, val);
+    load_products<T, G, false, kSteps>(p, ra, na, lane, col, val);
+    const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, p.lo[row], lane,
+                                               p.ranks + static_cast<int64_t>(row) * kBmrSlots);
+    if (lane == 0) p.c_rowptr[row + 1] = total;
+  }
+}
 
-    if constexpr (!NUMERIC) {
-      const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, p.lo[row], lane, ranks);
-      if (lane == 0) p.c_rowptr[row + 1] = total;
-    } else {
-      int rk[kSteps];
+// Numeric pass of the register bitmap rows.  A warp takes kHdrRows rows of
+// its share at a time: first the lanes fetch, for all of them together, the
+// row bounds, C's row offsets and every stored A entry with its B row extent
+// (a chain of dependent loads, paid once per batch instead of once per row);
+// then, row by row, every lane loads its products and their stored ranks in
+// one round of independent loads, the first product of every column stores
+// its column and value at its rank in a compact staging array, the products
+// that repeat a column add theirs (a shared-memory atomic, the atomic level
+// of Sec. 4), and the warp copies the sorted row to C with coalesced stores.
+constexpr int kHdrRows = 8;
+
+template <typename T>
+constexpr size_t numeric_warp_bytes() {
+  return static_cast<size_t>(kBmrCap) * (4 + sizeof(T)) +
+         static_cast<size_t>(kHdrRows) * kBmrMaxA * (sizeof(long long) + sizeof(int) + sizeof(T)) +
+         static_cast<size_t>(kHdrRows) * (2 * sizeof(long long) + sizeof(int));
+}
+
+template <typename T, int G>
+__global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_numeric_kernel(const RowPlan<T> p) {
+  constexpr int kGroups = 32 / G;
+  constexpr int kSteps = kBmrMaxA / kGroups;
+  constexpr int kEnt = kHdrRows * kBmrMaxA;
+  static_assert(kSteps % 2 == 0, "ranks are fetched in pairs of steps");
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int sub = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int grp = lane / G, gl = lane % G;
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * numeric_warp_bytes<T>();
+  int* st_key = reinterpret_cast<int*>(ws);
+  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kBmrCap) * 4);
+  long long* h_b0 = reinterpret_cast<long long*>(ws + static_cast<size_t>(kBmrCap) * (4 + sizeof(T)));
+  T* h_a = reinterpret_cast<T*>(h_b0 + kEnt);
+  int* h_len = reinterpret_cast<int*>(h_a + kEnt);
+  long long* h_cbase = reinterpret_cast<long long*>(h_len + kEnt);  // C offset and nnz of each batch row
+  long long* h_cnt = h_cbase + kHdrRows;
+  int* h_row = reinterpret_cast<int*>(h_cnt + kHdrRows);
+
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
+  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * kHdrRows; r0 < p.seg_len;
+       r0 += warps * kHdrRows) {
+    // Batch header: lane i < kHdrRows fetches row r0 + i.
+    int na_l = 0;
+    long long ra_l = 0;
+    if (lane < kHdrRows) {
+      int row_l = -1;
+      if (r0 + lane < p.seg_len) {
+        row_l = p.perm[p.seg_begin + r0 + lane];
+        ra_l = p.A.rowptr[row_l];
+        const long long na = p.A.rowptr[row_l + 1] - ra_l;
+        na_l = static_cast<int>(na < kBmrMaxA ? (na > 0 ? na : 0) : kBmrMaxA);
+        const long long cb = p.c_rowptr[row_l];
+        h_cbase[lane] = cb;
+        h_cnt[lane] = p.c_rowptr[row_l + 1] - cb;
+      }
+      h_row[lane] = row_l;
+    }
 #pragma unroll
-      for (int s = 0; s < kSteps; ++s) rk[s] = col[s] >= 0 ? ranks[(s << 5) | lane] : 0;
-      const int64_t cbase = p.c_rowptr[row];
-      const int64_t want = p.c_rowptr[row + 1] - cbase;
+    for (int q = 0; q < kEnt / 32; ++q) {
+      const int e = q * 32 + lane;
+      const int i = e / kBmrMaxA, j = e % kBmrMaxA;
+      const long long ra = __shfl_sync(kFull, ra_l, i);
+      const int na = __shfl_sync(kFull, na_l, i);
+      int len = 0;
+      if (j < na) {
+        const int k = p.A.colidx[ra + j];
+        const long long b0 = p.B.rowptr[k];
+        len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        h_b0[e] = b0;
+        h_a[e] = p.A.vals[ra + j];
+      }
+      h_len[e] = len;
+    }
+    __syncwarp();
+    for (int i = 0; i < kHdrRows; ++i) {
+      const int row = h_row[i];
+      if (row < 0) break;
+      const long long cbase = h_cbase[i];
+      const long long want = h_cnt[i];
       const int cnt = static_cast<int>(want < kBmrCap ? want : kBmrCap);  // staging bounds every access
       if (lane == 0 && want > kBmrCap) atomicOr(&p.sum->status, kErrCount);
-      // The first product of every column stores its value; the rare repeats add theirs after.
+      const uint32_t* ranks2 = reinterpret_cast<const uint32_t*>(p.ranks + static_cast<int64_t>(row) * kBmrSlots);
+      int col[kSteps];
+      uint32_t rk2[kSteps / 2];  // ranks of steps q (low half) and q + kSteps / 2 (high half)
+      T val[kSteps];
+      uint32_t has_lo = 0;  // bit q: step q has a product
+#pragma unroll
+      for (int st = 0; st < kSteps; ++st) {
+        const int e = i * kBmrMaxA + st * kGroups + grp;
+        const bool has = gl < h_len[e];
+        col[st] = -1;
+        val[st] = T(0);
+        if (has) {
+          const long long b0 = h_b0[e];
+          col[st] = p.B.colidx[b0 + gl];
+          val[st] = p.B.vals[b0 + gl];  // scaled by the A value at the scatter
+        }
+        if (st < kSteps / 2) {
+          has_lo |= static_cast<uint32_t>(has) << st;
+        } else {
+          const int q = st - kSteps / 2;
+          rk2[q] = (((has_lo >> q) & 1u) || has) ? ranks2[rank_word<kSteps>(q, lane)] : 0u;
+        }
+      }
       bool bad = false, repeats = false;
 #pragma unroll
-      for (int s = 0; s < kSteps; ++s) {
-        if (col[s] >= 0) {
-          const int r = rk[s] & 0x7fff;
+      for (int st = 0; st < kSteps; ++st) {
+        if (col[st] >= 0) {
+          const int rk = static_cast<int>(st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16);
+          const int r = rk & 0x7fff;
+          val[st] *= h_a[i * kBmrMaxA + st * kGroups + grp];
           if (r >= cnt) {
             bad = true;
-          } else if (rk[s] & 0x8000) {
+          } else if (rk & 0x8000) {
             repeats = true;
           } else {
-            st_key[r] = col[s];
-            st_val[r] = val[s];
+            st_key[r] = col[st];
+            st_val[r] = val[st];
           }
         }
       }
@@ -246,9 +355,10 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? (sizeof(T) == 8 ? 
       __syncwarp();
       if (__any_sync(kFull, repeats)) {
 #pragma unroll
-        for (int s = 0; s < kSteps; ++s) {
-          const int r = rk[s] & 0x7fff;
-          if (col[s] >= 0 && (rk[s] & 0x8000) && r < cnt) atomicAdd(&st_val[r], val[s]);
+        for (int st = 0; st < kSteps; ++st) {
+          const int rk = static_cast<int>(st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16);
+          const int r = rk & 0x7fff;
+          if (col[st] >= 0 && (rk & 0x8000) && r < cnt) atomicAdd(&st_val[r], val[st]);
         }
         __syncwarp();
       }
@@ -269,52 +379,73 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, NUMERIC ? (sizeof(T) == 8 ? 
 //
 // One CTA of kPlanThreads threads (two warps) works on one row, so the
 // bitmap of a row is shared by all of them: thread t owns the contiguous
-// words [t * WPT, (t + 1) * WPT), stored at (w % WPT) * kPlanThreads + w / WPT.  Product
-// (stored A entry j, element e of B[k_j,:]) keeps the slot j * G + e, the
-// same slot the one-warp numeric kernel uses.
-#ifndef WS_PLAN_THREADS
-#define WS_PLAN_THREADS 64
-#endif
-constexpr int kPlanThreads = WS_PLAN_THREADS;
+// words [t * WPT, (t + 1) * WPT) (bits of columns [32 t WPT, 32 (t + 1) WPT)).
+// After the product bits are set, every thread counts the bits of its own
+// words in one sweep (no search for the non-zero words: the sweep is
+// branch-free and, with 32 words per thread, reads them as eight 16-byte
+// chunks), the CTA scans the counts, and every thread stores the rank of
+// the first column of each of its words.  A product's rank is then that word
+// rank plus the bits below it in its word.
+constexpr int kPlanThreads = 64;
 
 template <int LOGW>
 struct PlanShape {
   static constexpr int kWords = 1 << LOGW;
   static constexpr int kWPT = kWords >= kPlanThreads ? kWords / kPlanThreads : 1;  // words per thread
-  static constexpr int kLogThreads = kPlanThreads == 64 ? 6 : kPlanThreads == 128 ? 7 : 8;
-  static constexpr int kLogWPT = LOGW >= kLogThreads ? LOGW - kLogThreads : 0;
+  static constexpr int kLogWPT = LOGW >= 6 ? LOGW - 6 : 0;
   static constexpr int kPhysWords = kWPT * kPlanThreads;
-  static constexpr int kSPT = kWPT >= 32 ? kWPT / 32 : 1;  // summary words per thread
-  static constexpr size_t bytes() {
-    return static_cast<size_t>(kPhysWords) * 6 + kPlanThreads * 4 + static_cast<size_t>(kSPT) * kPlanThreads * 4;
-  }
+  // 32 words per thread: thread-major rows of eight 16-byte chunks, chunk c of
+  // thread t at position c ^ (t % 8), so the eight threads of a quarter warp
+  // read eight different bank groups.  Fewer: word i of thread t at i * 64 + t.
+  static constexpr bool kVec = kWPT == 32;
+  static constexpr size_t bytes() { return static_cast<size_t>(kPhysWords) * 6; }  // bitmap + uint16 word ranks
 };
+static_assert(kPlanThreads == 64, "the shapes below assume 64 threads");
+// 16 CTAs per SM (the shared-memory limit): 64 registers a thread.
+constexpr int kPlanMinBlocks = 16;
 
 template <class S>
 __device__ __forceinline__ uint32_t plan_phys(uint32_t w) {
-  return (w & (S::kWPT - 1)) * kPlanThreads + (w >> S::kLogWPT);
+  if constexpr (S::kVec) {
+    const uint32_t t = w >> 5, i = w & 31u;
+    return (t << 5) | (((i >> 2) ^ (t & 7u)) << 2) | (i & 3u);
+  } else {
+    return (w & (S::kWPT - 1)) * kPlanThreads + (w >> S::kLogWPT);
+  }
+}
+
+// Position of word w's rank in the uint16 rank array: for 32 words per thread,
+// thread-major rows of four 16-byte chunks (eight ranks each), chunk q of
+// thread t at position q ^ ((t / 2) % 4) (a conflict-free 16-byte store per
+// quarter warp); otherwise the bitmap's layout.
+template <class S>
+__device__ __forceinline__ uint32_t plan_pre(uint32_t w) {
+  if constexpr (S::kVec) {
+    const uint32_t t = w >> 5, i = w & 31u;
+    return (t << 5) | (((i >> 3) ^ ((t >> 1) & 3u)) << 3) | (i & 7u);
+  } else {
+    return plan_phys<S>(w);
+  }
 }
 
 template <typename T, int LOGW, int G>
-__global__ void __launch_bounds__(kPlanThreads, 1024 / kPlanThreads) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
+__global__ void __launch_bounds__(kPlanThreads, kPlanMinBlocks) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
                                                                 int64_t ncols, int32_t* pending) {
   using S = PlanShape<LOGW>;
   constexpr int kGroups = kPlanThreads / G;   // A entries per step
   constexpr int kSteps = (kBmrMaxA + kGroups - 1) / kGroups;  // steps covering kBmrMaxA entries
+  constexpr int kW = kPlanThreads / 32;
+  constexpr int kLoc = (S::kWPT + 1) / 2;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint32_t* bm = reinterpret_cast<uint32_t*>(smem_raw);
   uint16_t* pre = reinterpret_cast<uint16_t*>(smem_raw + static_cast<size_t>(S::kPhysWords) * 4);
-  int* base = reinterpret_cast<int*>(smem_raw + static_cast<size_t>(S::kPhysWords) * 6);
-  uint32_t* sm = reinterpret_cast<uint32_t*>(base + kPlanThreads);
   __shared__ long long s_b0[kBmrMaxA];
   __shared__ int s_len[kBmrMaxA];
-  __shared__ int s_red[2 * (kPlanThreads / 32)];
-  __shared__ long long s_scan[32];
+  __shared__ int s_red[2 * kW];
   const int t = threadIdx.x;
   const int lane = t & 31, warp = t >> 5;
   const int grp = t / G, gl = t % G;
   for (int i = t; i < S::kPhysWords; i += kPlanThreads) bm[i] = 0u;
-  for (int i = t; i < S::kSPT * kPlanThreads; i += kPlanThreads) sm[i] = 0u;
   __syncthreads();
   const long long words = (ncols + 31) >> 5;
   int taken = 0;
@@ -340,7 +471,6 @@ __global__ void __launch_bounds__(kPlanThreads, 1024 / kPlanThreads) bmr_plan_ke
         ub += __shfl_xor_sync(kFull, ub, o);
         mx = max(mx, __shfl_xor_sync(kFull, mx, o));
       }
-      constexpr int kW = kPlanThreads / 32;
       if (lane == 0) {
         s_red[warp] = ub;
         s_red[kW + warp] = mx;
@@ -368,46 +498,118 @@ __global__ void __launch_bounds__(kPlanThreads, 1024 / kPlanThreads) bmr_plan_ke
         for (int st = 0; st < kSteps; ++st) {
           if (col[st] >= 0) {
             const uint32_t off = static_cast<uint32_t>(col[st]);
-            const uint32_t w = off >> 5;
-            const uint32_t jw = w & (S::kWPT - 1);
             const uint32_t bit = 1u << (off & 31u);
-            if (atomicOr(bm + plan_phys<S>(w), bit) & bit) dup |= 1u << st;
-            atomicOr(sm + (jw >> 5) * kPlanThreads + (w >> S::kLogWPT), 1u << (jw & 31u));
+            if (atomicOr(bm + plan_phys<S>(off >> 5), bit) & bit) dup |= 1u << st;
           }
         }
         __syncthreads();
+        // Sweep: local rank of the first column of each of this thread's words,
+        // two per register (word 2k low half, 2k + 1 high half).
+        uint32_t loc[kLoc];
         int run = 0;
+        if constexpr (S::kVec) {
+          const uint4* mine = reinterpret_cast<const uint4*>(bm + t * 32);
 #pragma unroll
-        for (int h = 0; h < S::kSPT; ++h) {
-          uint32_t m = sm[h * kPlanThreads + t];
-          sm[h * kPlanThreads + t] = 0u;  // only this thread reads it
-          while (m) {
-            const int b = __ffs(m) - 1;
-            m &= m - 1u;
-            const int ph = ((h << 5) | b) * kPlanThreads + t;
-            pre[ph] = static_cast<uint16_t>(run);
-            run += __popc(bm[ph]);
+          for (int c = 0; c < 8; ++c) {
+            const uint4 v = mine[c ^ (t & 7)];
+            loc[2 * c] = static_cast<uint32_t>(run);
+            run += __popc(v.x);
+            loc[2 * c] |= static_cast<uint32_t>(run) << 16;
+            run += __popc(v.y);
+            loc[2 * c + 1] = static_cast<uint32_t>(run);
+            run += __popc(v.z);
+            loc[2 * c + 1] |= static_cast<uint32_t>(run) << 16;
+            run += __popc(v.w);
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < S::kWPT; ++i) {
+            const int pc = __popc(bm[i * kPlanThreads + t]);
+            if (i & 1) {
+              loc[i >> 1] |= static_cast<uint32_t>(run) << 16;
+            } else {
+              loc[i >> 1] = static_cast<uint32_t>(run);
+            }
+            run += pc;
           }
         }
-        long long total;
-        base[t] = static_cast<int>(block_exclusive_scan(static_cast<long long>(run), s_scan, &total));
+        // Exclusive scan of the per-thread counts in thread order (= column order).
+        int incl = run;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(kFull, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (lane == 31) s_red[warp] = incl;
         __syncthreads();
-        uint16_t* ranks = p.ranks + row * kBmrSlots;
+        int before = 0, total = 0;
+#pragma unroll
+        for (int w2 = 0; w2 < kW; ++w2) {
+          const int v = s_red[w2];
+          before += w2 < warp ? v : 0;
+          total += v;
+        }
+        // Word ranks = thread base + local ranks (both halves: no carry, every rank <= kBmrCap).
+        const uint32_t base = static_cast<uint32_t>(before + incl - run);
+        const uint32_t base2 = base | (base << 16);
+        if constexpr (S::kVec) {
+          uint4* mine = reinterpret_cast<uint4*>(pre + t * 32);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            mine[q ^ ((t >> 1) & 3)] =
+                make_uint4(loc[4 * q] + base2, loc[4 * q + 1] + base2, loc[4 * q + 2] + base2, loc[4 * q + 3] + base2);
+        } else {
+#pragma unroll
+          for (int i = 0; i < S::kWPT; ++i)
+            pre[i * kPlanThreads + t] = static_cast<uint16_t>(((loc[i >> 1] >> (16 * (i & 1))) & 0xffffu) + base);
+        }
+        __syncthreads();
+        int rk[kSteps];
 #pragma unroll
         for (int st = 0; st < kSteps; ++st) {
+          rk[st] = 0;
           if (col[st] >= 0) {
             const uint32_t off = static_cast<uint32_t>(col[st]);
             const uint32_t w = off >> 5;
-            const uint32_t ph = plan_phys<S>(w);
-            const int pos = base[w >> S::kLogWPT] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
+            rk[st] = (pre[plan_pre<S>(w)] + __popc(bm[plan_phys<S>(w)] & ((1u << (off & 31u)) - 1u))) |
+                     static_cast<int>(((dup >> st) & 1u) << 15);
+          }
+        }
+        // Stored A entry j of this thread at step st is j = st * kGroups + grp;
+        // in the one-warp numeric kernel it sits at step j / kNumGroups of
+        // lane (j % kNumGroups) * G + gl.
+        constexpr int kNumGroups = 32 / G;
+        constexpr int kNumSteps = kBmrMaxA / kNumGroups;
+        if constexpr (8 % kGroups == 0) {
+          // entries j and j + 8 (steps st and st + kPair) share one rank word
+          constexpr int kPair = 8 / kGroups;
+          uint32_t* ranks32 = reinterpret_cast<uint32_t*>(p.ranks + row * kBmrSlots);
+#pragma unroll
+          for (int st = 0; st < kPair; ++st) {
             const int j = st * kGroups + grp;
-            ranks[j * G + gl] = static_cast<uint16_t>(pos | (((dup >> st) & 1u) << 15));
+            if (col[st] >= 0 || col[st + kPair] >= 0)
+              ranks32[rank_word<kNumSteps>(j / kNumGroups, (j % kNumGroups) * G + gl)] = rank_pack(rk[st], rk[st + kPair]);
+          }
+        } else {
+          uint16_t* ranks = p.ranks + row * kBmrSlots;
+#pragma unroll
+          for (int st = 0; st < kSteps; ++st) {
+            const int j = st * kGroups + grp;
+            const int sn = j / kNumGroups;
+            if (col[st] >= 0)
+              ranks[2 * rank_word<kNumSteps>(sn, (j % kNumGroups) * G + gl) + (sn >= kNumSteps / 2)] =
+                  static_cast<uint16_t>(rk[st]);
           }
         }
         __syncthreads();
+        // Clear this thread's words (conflict-free).
+        if constexpr (S::kVec) {
+          uint4* mine = reinterpret_cast<uint4*>(bm + t * 32);
 #pragma unroll
-        for (int st = 0; st < kSteps; ++st) {
-          if (col[st] >= 0) bm[plan_phys<S>(static_cast<uint32_t>(col[st]) >> 5)] = 0u;
+          for (int c = 0; c < 8; ++c) mine[c ^ (t & 7)] = make_uint4(0u, 0u, 0u, 0u);  // same order as the sweep
+        } else {
+#pragma unroll
+          for (int i = 0; i < S::kWPT; ++i) bm[i * kPlanThreads + t] = 0u;
         }
         if (t == 0) {
           p.c_rowptr[row + 1] = total;
@@ -443,13 +645,20 @@ int64_t clamp_grid(int64_t want, int num_sms, int per_sm) {
 
 template <typename T, int LOGW, int G>
 void launch_bmr_g(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s) {
-  using S = BmrShape<LOGW>;
-  const size_t smem = static_cast<size_t>(kRowsPerCta) * S::template warp_bytes<T>(numeric);
-  auto kern = numeric ? bmr_rows_kernel<T, LOGW, G, true> : bmr_rows_kernel<T, LOGW, G, false>;
-  static int per_sm[2] = {0, 0};
-  if (per_sm[numeric] == 0) per_sm[numeric] = occupancy(kern, 32 * kRowsPerCta, smem);
-  const int64_t grid = clamp_grid((p.seg_len + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm[numeric]);
-  kern<<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
+  if (numeric) {
+    const size_t smem = static_cast<size_t>(kRowsPerCta) * numeric_warp_bytes<T>();
+    static int per_sm = 0;
+    if (per_sm == 0) per_sm = occupancy(bmr_numeric_kernel<T, G>, 32 * kRowsPerCta, smem);
+    const int64_t per_cta = static_cast<int64_t>(kRowsPerCta) * kHdrRows;
+    const int64_t grid = clamp_grid((p.seg_len + per_cta - 1) / per_cta, num_sms, per_sm);
+    bmr_numeric_kernel<T, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
+    return;
+  }
+  const size_t smem = static_cast<size_t>(kRowsPerCta) * BmrShape<LOGW>::bytes();
+  static int per_sm = 0;
+  if (per_sm == 0) per_sm = occupancy(bmr_symbolic_kernel<T, LOGW, G>, 32 * kRowsPerCta, smem);
+  const int64_t grid = clamp_grid((p.seg_len + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm);
+  bmr_symbolic_kernel<T, LOGW, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
 }
 
 template <typename T, int LOGW>
