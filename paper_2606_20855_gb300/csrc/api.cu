@@ -115,6 +115,7 @@ struct Plan {
   int64_t n_sort = 0, n_empty = 0, dense_slices = 0, products = 0;
   int log2_group = 5;
   int wide_bin = 2;  // register bitmap bin of the rows counted by the planning pass
+  bool all_planned = false;  // the planning pass took every row: its segment is rows 0..m-1 in order
   int dense_width = 0;
   int run_limit = 64;
   int sym_launches = 0, num_launches = 0;
@@ -232,58 +233,14 @@ ws_status_t carve_slices(Plan* pl, int64_t nslices, cudaStream_t s) {
   return WS_OK;
 }
 
+// Second half of the symbolic pass when some rows were not ranked by the
+// planning pass: group the rows by segment, run the per-bin symbolic kernels,
+// scan the counts into C's row pointer and read the summary back.
 template <typename T>
-ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, cudaStream_t s,
-                          int64_t* nnz_out) {
+ws_status_t symbolic_bins(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, RowPlan<T> p, int64_t off,
+                          int sms, cudaStream_t s) {
   const int64_t m = A->nrows;
-  const int dev = C->device;
-  const int sms = num_sms_of(dev);
-  pl->ready = false;
-  pl->sym_launches = 0;
-  pl->log2_group = log2_group_for(B);
-  pl->run_limit = g_run_limit;
-  pl->dense_width = g_dense_width > 0 ? g_dense_width : (sizeof(T) == 8 ? 8192 : 16384);
-
-  ws_status_t st = carve_rows(pl, m, s);
-  if (st != WS_OK) return st;
-  WS_CUDA(cudaMemsetAsync(pl->dsum, 0, sizeof(DevSummary), s), "cudaMemsetAsync(summary)");
-  WS_CUDA(cudaMemsetAsync(C->rowptr, 0, sizeof(int64_t), s), "cudaMemsetAsync(rowptr[0])");
-
-  RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
-  if (m > 0) {
-    AnalyzeParams ap{m,           g_hash_max, g_bitmap_span,   1 << pl->log2_group, g_bmr_max_a,
-                     g_rcd_max_a, g_wb_span,  pl->dense_width, kLongRowThreshold};
-    // When every row of C fits the widest register bitmap (B has at most
-    // 65,536 columns), the planning pass counts the eligible rows in its first
-    // read of A and only the remaining rows go through the analysis kernel.
-    const bool plan_pass = g_bmr_max_a > 0 && B->ncols > 0 && B->ncols <= kMaxBitmapSpan && g_bitmap_span >= B->ncols;
-    pl->wide_bin = bmr_bin_for_span(B->ncols);
-    if (plan_pass) {
-      st = pl->ranks.reserve(static_cast<size_t>(m) * kBmrSlots * sizeof(uint16_t), s);
-      if (st != WS_OK) return st;
-      p.ranks = static_cast<uint16_t*>(pl->ranks.ptr);
-      launch_bmr_plan<T>(p, ap, B->ncols, pl->pending, sms, s, &pl->sym_launches);
-      launch_analyze<T>(p, ap, pl->long_rows, pl->pending, sms, s, &pl->sym_launches);
-    } else {
-      launch_analyze<T>(p, ap, pl->long_rows, nullptr, sms, s, &pl->sym_launches);
-    }
-    WS_CUDA(cudaGetLastError(), "analyze launch");
-  }
-  st = read_summary(pl, s);
-  if (st != WS_OK) return st;
-  const DevSummary& hs = *pl->host_sum;
-  int64_t off = 0;
-  for (int g = 0; g < kNumSegs; ++g) {
-    pl->seg_count[g] = hs.seg_count[g];
-    pl->seg_offset[g] = off;
-    off += hs.seg_count[g];
-  }
-  pl->seg_offset[kNumSegs] = off;
-  pl->n_empty = hs.n_empty;
-  pl->products = hs.products;
-  pl->dense_slices = hs.dense_slices;
-  if (pl->dense_slices > INT32_MAX) return fail(WS_ERR_OVERFLOW, "too many dense-window slices (%lld)", (long long)pl->dense_slices);
-
+  ws_status_t st = WS_OK;
   if (off > 0) {
     launch_scatter<T>(p, m, pl->seg_offset, sms, s, &pl->sym_launches);
   }
@@ -338,6 +295,68 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
   WS_CUDA(cudaGetLastError(), "symbolic launches");
   st = read_summary(pl, s);
   if (st != WS_OK) return st;
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, cudaStream_t s,
+                          int64_t* nnz_out) {
+  const int64_t m = A->nrows;
+  const int dev = C->device;
+  const int sms = num_sms_of(dev);
+  pl->ready = false;
+  pl->sym_launches = 0;
+  pl->log2_group = log2_group_for(B);
+  pl->run_limit = g_run_limit;
+  pl->dense_width = g_dense_width > 0 ? g_dense_width : (sizeof(T) == 8 ? 8192 : 16384);
+
+  ws_status_t st = carve_rows(pl, m, s);
+  if (st != WS_OK) return st;
+  WS_CUDA(cudaMemsetAsync(pl->dsum, 0, sizeof(DevSummary), s), "cudaMemsetAsync(summary)");
+  WS_CUDA(cudaMemsetAsync(C->rowptr, 0, sizeof(int64_t), s), "cudaMemsetAsync(rowptr[0])");
+
+  RowPlan<T> p = make_rowplan<T>(A, B, C, pl);
+  if (m > 0) {
+    AnalyzeParams ap{m,           g_hash_max, g_bitmap_span,   1 << pl->log2_group, g_bmr_max_a,
+                     g_rcd_max_a, g_wb_span,  pl->dense_width, kLongRowThreshold};
+    // When every row of C fits the widest register bitmap (B has at most
+    // 65,536 columns), the planning pass counts the eligible rows in its first
+    // read of A and only the remaining rows go through the analysis kernel.
+    const bool plan_pass = g_bmr_max_a > 0 && B->ncols > 0 && B->ncols <= kMaxBitmapSpan && g_bitmap_span >= B->ncols;
+    pl->wide_bin = bmr_bin_for_span(B->ncols);
+    if (plan_pass) {
+      st = pl->ranks.reserve(static_cast<size_t>(m) * kBmrSlots * sizeof(uint16_t), s);
+      if (st != WS_OK) return st;
+      p.ranks = static_cast<uint16_t*>(pl->ranks.ptr);
+      launch_bmr_plan<T>(p, ap, B->ncols, pl->pending, sms, s, &pl->sym_launches);
+      launch_analyze<T>(p, ap, pl->long_rows, pl->pending, sms, s, &pl->sym_launches);
+      // If the planning pass took every row, all counts are in place now: a
+      // scan queued here (a no-op otherwise) saves the second read-back.
+      launch_scan(C->rowptr, m, pl->partials, pl->dsum, s, &pl->sym_launches, &pl->dsum->n_pending);
+    } else {
+      launch_analyze<T>(p, ap, pl->long_rows, nullptr, sms, s, &pl->sym_launches);
+    }
+    WS_CUDA(cudaGetLastError(), "analyze launch");
+  }
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  const DevSummary& hs = *pl->host_sum;
+  int64_t off = 0;
+  for (int g = 0; g < kNumSegs; ++g) {
+    pl->seg_count[g] = hs.seg_count[g];
+    pl->seg_offset[g] = off;
+    off += hs.seg_count[g];
+  }
+  pl->seg_offset[kNumSegs] = off;
+  pl->n_empty = hs.n_empty;
+  pl->products = hs.products;
+  pl->dense_slices = hs.dense_slices;
+  if (pl->dense_slices > INT32_MAX) return fail(WS_ERR_OVERFLOW, "too many dense-window slices (%lld)", (long long)pl->dense_slices);
+  pl->all_planned = m > 0 && hs.n_pending == 0 && pl->seg_count[kSegBmrWide] == m;
+  if (!pl->all_planned) {
+    st = symbolic_bins<T>(A, B, C, pl, p, off, sms, s);
+    if (st != WS_OK) return st;
+  }
   st = device_status(*pl->host_sum);
   if (st != WS_OK) return st;
   pl->n_sort = pl->host_sum->n_sort;
@@ -364,7 +383,9 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
   if (pl->seg_count[kSegBmrWide] > 0) {
     p.seg_begin = pl->seg_offset[kSegBmrWide];
     p.seg_len = pl->seg_count[kSegBmrWide];
+    if (pl->all_planned) p.perm = nullptr;  // rows in order, no permutation was built
     launch_bmr<T>(p, pl->wide_bin, true, sms, s, &pl->num_launches);
+    p.perm = pl->perm;
   }
   if (pl->seg_count[kSegRcd] > 0) {
     p.seg_begin = pl->seg_offset[kSegRcd];

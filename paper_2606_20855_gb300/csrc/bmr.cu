@@ -277,7 +277,7 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
     if (lane < kHdrRows) {
       int row_l = -1;
       if (r0 + lane < p.seg_len) {
-        row_l = p.perm[p.seg_begin + r0 + lane];
+        row_l = p.perm ? p.perm[p.seg_begin + r0 + lane] : static_cast<int>(p.seg_begin + r0 + lane);
         ra_l = p.A.rowptr[row_l];
         const long long na = p.A.rowptr[row_l + 1] - ra_l;
         na_l = static_cast<int>(na < kBmrMaxA ? (na > 0 ? na : 0) : kBmrMaxA);
@@ -392,7 +392,6 @@ template <int LOGW>
 struct PlanShape {
   static constexpr int kWords = 1 << LOGW;
   static constexpr int kWPT = kWords >= kPlanThreads ? kWords / kPlanThreads : 1;  // words per thread
-  static constexpr int kLogWPT = LOGW >= 6 ? LOGW - 6 : 0;
   static constexpr int kPhysWords = kWPT * kPlanThreads;
   // 32 words per thread: thread-major rows of eight 16-byte chunks, chunk c of
   // thread t at position c ^ (t % 8), so the eight threads of a quarter warp
@@ -407,10 +406,10 @@ constexpr int kPlanMinBlocks = 16;
 template <class S>
 __device__ __forceinline__ uint32_t plan_phys(uint32_t w) {
   if constexpr (S::kVec) {
-    const uint32_t t = w >> 5, i = w & 31u;
-    return (t << 5) | (((i >> 2) ^ (t & 7u)) << 2) | (i & 3u);
+    // thread t = w / 32, word i = w % 32: chunk bits (2..4) of w XOR t % 8 (bits 5..7)
+    return w ^ ((w >> 3) & 0x1cu);
   } else {
-    return (w & (S::kWPT - 1)) * kPlanThreads + (w >> S::kLogWPT);
+    return (w % S::kWPT) * kPlanThreads + w / S::kWPT;
   }
 }
 
@@ -421,8 +420,8 @@ __device__ __forceinline__ uint32_t plan_phys(uint32_t w) {
 template <class S>
 __device__ __forceinline__ uint32_t plan_pre(uint32_t w) {
   if constexpr (S::kVec) {
-    const uint32_t t = w >> 5, i = w & 31u;
-    return (t << 5) | (((i >> 3) ^ ((t >> 1) & 3u)) << 3) | (i & 7u);
+    // chunk bits (3..4) of w XOR (t / 2) % 4 (bits 6..7)
+    return w ^ ((w >> 3) & 0x18u);
   } else {
     return plan_phys<S>(w);
   }

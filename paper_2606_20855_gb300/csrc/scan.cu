@@ -5,7 +5,9 @@
 //
 // Reduce-then-scan in three launches (tile sums, scan of the tile sums in one
 // CTA, scan of each tile plus its offset).  No CTA waits on another, so the
-// scan cannot stall however the CTAs are scheduled.
+// scan cannot stall however the CTAs are scheduled.  With a `skip` flag the
+// three kernels do nothing when *skip != 0 (a scan queued before the host
+// knows whether every count is in place).
 #include "ws_internal.cuh"
 
 namespace wsk {
@@ -16,7 +18,9 @@ constexpr int kScanThreads = 256;
 constexpr int kScanItems = 16;
 constexpr int kTile = kScanThreads * kScanItems;
 
-__global__ void __launch_bounds__(kScanThreads) scan_reduce_kernel(const int64_t* x, int64_t n, int64_t* partial) {
+__global__ void __launch_bounds__(kScanThreads) scan_reduce_kernel(const int64_t* x, int64_t n, int64_t* partial,
+                                                                    const int* skip) {
+  if (skip && *skip) return;
   __shared__ long long scratch[32];
   const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
   long long s = 0;
@@ -30,7 +34,8 @@ __global__ void __launch_bounds__(kScanThreads) scan_reduce_kernel(const int64_t
 }
 
 // Exclusive scan of the tile sums, in place, by one CTA of 1024 threads.
-__global__ void __launch_bounds__(1024) scan_partials_kernel(int64_t* partial, int64_t nb) {
+__global__ void __launch_bounds__(1024) scan_partials_kernel(int64_t* partial, int64_t nb, const int* skip) {
+  if (skip && *skip) return;
   __shared__ long long scratch[32];
   long long carry = 0;
   for (int64_t b0 = 0; b0 < nb; b0 += blockDim.x) {
@@ -44,7 +49,8 @@ __global__ void __launch_bounds__(1024) scan_partials_kernel(int64_t* partial, i
 }
 
 __global__ void __launch_bounds__(kScanThreads) scan_apply_kernel(int64_t* x, int64_t n, const int64_t* partial,
-                                                                   DevSummary* sum) {
+                                                                   DevSummary* sum, const int* skip) {
+  if (skip && *skip) return;
   __shared__ long long scratch[32];
   const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
   // Each thread owns kScanItems consecutive elements.
@@ -70,12 +76,13 @@ __global__ void __launch_bounds__(kScanThreads) scan_apply_kernel(int64_t* x, in
 
 int64_t scan_partials_needed(int64_t m) { return (m + kTile - 1) / kTile; }
 
-void launch_scan(int64_t* rowptr, int64_t m, int64_t* partials, DevSummary* sum, cudaStream_t s, int* launches) {
+void launch_scan(int64_t* rowptr, int64_t m, int64_t* partials, DevSummary* sum, cudaStream_t s, int* launches,
+                 const int* skip) {
   if (m <= 0) return;
   const int64_t nb = scan_partials_needed(m);
-  scan_reduce_kernel<<<static_cast<int>(nb), kScanThreads, 0, s>>>(rowptr + 1, m, partials);
-  scan_partials_kernel<<<1, 1024, 0, s>>>(partials, nb);
-  scan_apply_kernel<<<static_cast<int>(nb), kScanThreads, 0, s>>>(rowptr + 1, m, partials, sum);
+  scan_reduce_kernel<<<static_cast<int>(nb), kScanThreads, 0, s>>>(rowptr + 1, m, partials, skip);
+  scan_partials_kernel<<<1, 1024, 0, s>>>(partials, nb, skip);
+  scan_apply_kernel<<<static_cast<int>(nb), kScanThreads, 0, s>>>(rowptr + 1, m, partials, sum, skip);
   *launches += 3;
 }
 

@@ -191,7 +191,9 @@ void launch_direct(const RowPlan<T>& p, int num_sms, cudaStream_t s, int* launch
 template <typename T>
 void launch_sort(const RowPlan<T>& p, int64_t nrows, int num_sms, cudaStream_t s, int* launches);
 
-void launch_scan(int64_t* rowptr, int64_t m, int64_t* partials, DevSummary* sum, cudaStream_t s, int* launches);
+// skip != nullptr: the scan does nothing when *skip != 0 (read on the device).
+void launch_scan(int64_t* rowptr, int64_t m, int64_t* partials, DevSummary* sum, cudaStream_t s, int* launches,
+                 const int* skip = nullptr);
 int64_t scan_partials_needed(int64_t m);
 
 void launch_validate(const int64_t* rowptr, const int32_t* colidx, int64_t nrows, int64_t ncols, int64_t nnz,
