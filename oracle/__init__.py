@@ -1,4 +1,4 @@
-"""CPU oracle for C = A*B on CSR matrices -- TEST INFRASTRUCTURE.
+"""CPU oracles for C = A*B and for C = A op B (elementwise) on CSR matrices -- TEST INFRASTRUCTURE.
 
 Only the tests, the smoke check and the benchmark's CPU-baseline leg use this
 package.  The CUDA library never imports or links it, and it imports nothing
@@ -8,7 +8,8 @@ from the CUDA library.
 C (all rows when ``rows`` is None) as numpy arrays computed by
 ``spgemm_oracle.cpp`` (Gustavson's row-wise algorithm with an ordered map per
 row, Sec. 5.1), with values accumulated in float64, plus
-absmass = sum |a*b| per output entry.
+absmass = sum |a*b| per output entry.  ``oracle_ewise(A, B, op)`` (ewise.py)
+is the elementwise SpAdd / Hadamard oracle.
 """
 from __future__ import annotations
 
@@ -99,4 +100,6 @@ def oracle_spgemm(A, B, rows=None, threads: int = 1) -> OracleCSR:
     return OracleCSR(nsel, B.ncols, rowptr, colidx, vals, absmass)
 
 
-__all__ = ["oracle_spgemm", "OracleCSR", "build", "LIB"]
+from .ewise import oracle_ewise  # noqa: E402  (needs OracleCSR above)
+
+__all__ = ["oracle_spgemm", "oracle_ewise", "OracleCSR", "build", "LIB"]

@@ -3,4 +3,5 @@
 Holds input generation only; no part of the sparse product is computed here.
 """
 from .matrices import *  # noqa: F401,F403
-from .matrices import HostCSR, WORKLOADS, WORKLOAD_ORDER, row_subset, workload  # noqa: F401
+from .matrices import (EWISE_WORKLOADS, HostCSR, WORKLOADS, WORKLOAD_ORDER, ewise_workload,  # noqa: F401
+                       permute_symmetric, row_subset, workload)

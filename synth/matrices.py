@@ -44,6 +44,9 @@ __all__ = [
     "random_csr",
     "workload",
     "WORKLOADS",
+    "permute_symmetric",
+    "ewise_workload",
+    "EWISE_WORKLOADS",
 ]
 
 
@@ -236,6 +239,41 @@ def workload(name: str):
         B = uniform_csr(1 << 20, 1 << 20, 4, rng, np.float64, "pos")
         return A, B
     raise KeyError(f"unknown workload {name!r}; known: {WORKLOAD_ORDER}")
+
+
+def permute_symmetric(A: HostCSR, perm: np.ndarray) -> HostCSR:
+    """P A P^T for a square A: entry (i, j) moves to (perm[i], perm[j]) with its value."""
+    if A.nrows != A.ncols:
+        raise ValueError("symmetric permutation needs a square matrix")
+    perm = np.asarray(perm, dtype=np.int64)
+    rows = perm[np.repeat(np.arange(A.nrows, dtype=np.int64), np.diff(A.rowptr))]
+    cols = perm[A.colidx.astype(np.int64)]
+    order = np.argsort(rows * A.ncols + cols, kind="stable")
+    rowptr = np.zeros(A.nrows + 1, dtype=np.int64)
+    np.cumsum(np.bincount(rows, minlength=A.nrows), out=rowptr[1:])
+    return HostCSR(A.nrows, A.ncols, rowptr, cols[order].astype(np.int32), A.vals[order])
+
+
+# Inputs of the elementwise operations C = A + B and C = A .* B: a power-law
+# graph standing in for the SNAP matrices, in the two cases the elementwise
+# benchmarks use -- B a randomly relabelled copy of A, and B = A.
+EWISE_WORKLOADS = {
+    "ewise_rmat20_perm": "R-MAT 2^20, edge factor 8, (a,b,c,d)=(.57,.19,.19,.05), fp64 values in (0,1], "
+                         "seed 4; B = P A P^T for a seeded random permutation P",
+    "ewise_rmat20_same": "the same R-MAT A (seed 4) with B = A",
+}
+
+
+def ewise_workload(name: str):
+    """Return (A, B) for a named elementwise workload."""
+    if name not in EWISE_WORKLOADS:
+        raise KeyError(f"unknown elementwise workload {name!r}; known: {list(EWISE_WORKLOADS)}")
+    rng = np.random.default_rng(4)
+    rp, ci, _ = rmat_pattern(20, 8, RMAT_PROBS, rng)
+    A = HostCSR(1 << 20, 1 << 20, rp, ci, _draw_values(rng, ci.size, "pos").astype(np.float64))
+    if name == "ewise_rmat20_same":
+        return A, A
+    return A, permute_symmetric(A, rng.permutation(A.nrows))
 
 
 def row_subset(A: HostCSR, rows: np.ndarray) -> HostCSR:
