@@ -66,7 +66,7 @@ typedef enum {
   WS_OK = 0,
   WS_ERR_INVALID_ARG = 1, /* NULL handle/pointer, negative size, bad enum        */
   WS_ERR_INVALID_CSR = 2, /* validation found broken CSR invariants              */
-  WS_ERR_SHAPE = 3,       /* A.ncols != B.nrows, or C is not A.nrows x B.ncols     */
+  WS_ERR_SHAPE = 3,       /* operand or output shapes do not fit the operation    */
   WS_ERR_DTYPE = 4,       /* A, B and C do not share one value type              */
   WS_ERR_OVERFLOW = 5,    /* a size exceeds what the index types can hold         */
   WS_ERR_ALLOC = 6,       /* device or pinned-host allocation failed             */
@@ -123,9 +123,49 @@ ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_
 ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
                               ws_stream_t stream);
 
+/* Elementwise operations (Sec. 5.2, "Sparse Linear Algebra": C = A op B). */
+typedef enum {
+  WS_EWISE_ADD = 1, /* SpAdd: C = A + B on the union of the two patterns            */
+  WS_EWISE_MUL = 2  /* Hadamard product: C = A .* B on the intersection of the two */
+} ws_ewise_op_t;
+
+/*
+ * ws_ewise_symbolic -- structure pass of the elementwise operation C = A op B
+ * (Sec. 5.2, "Sparse Linear Algebra", where SpAdd and the Hadamard product
+ * use the sharded sparse list: distinct rows of C go to distinct workers).
+ *   op   WS_EWISE_ADD: C holds (i, j) iff A or B stores (i, j), with
+ *        C[i,j] = A[i,j] + B[i,j] (a missing entry contributes nothing; a sum
+ *        of exactly 0.0 is kept);
+ *        WS_EWISE_MUL: C holds (i, j) iff both store (i, j), with
+ *        C[i,j] = A[i,j] * B[i,j].
+ * A and B have the same shape and dtype; C is an output handle of that shape
+ * and dtype.  Writes C.rowptr into the rowptr array of C's handle and returns
+ * nnz(C) in *nnz_out (host pointer).  Work is queued on `stream` and the call
+ * synchronises it (the caller needs nnz(C) to allocate C).  The chunk plan
+ * (rows cut into pieces of their merged column lists) is kept in C's handle
+ * for ws_ewise_numeric; device scratch is allocated stream-ordered on
+ * `stream` and cached in the handle.  Errors: WS_ERR_SHAPE, WS_ERR_DTYPE,
+ * WS_ERR_INVALID_ARG (NULL pointer, unknown op), WS_ERR_DEVICE (a kernel found
+ * inconsistent input, e.g. unsorted columns).
+ */
+ws_status_t ws_ewise_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int op, int64_t* nnz_out, ws_stream_t stream);
+
+/*
+ * ws_ewise_numeric -- value pass of C = A op B.
+ *   c_colidx  device int32[nnz(C)] written with C's column indices
+ *   c_vals    device value array [nnz(C)] of C's dtype
+ * Requires a completed ws_ewise_symbolic for the same A, B and C (A and B
+ * unchanged since).  Asynchronous on `stream`; device-side failures are
+ * reported by ws_spgemm_wait.  Values are computed in the value type: one
+ * rounding per entry.
+ */
+ws_status_t ws_ewise_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                             ws_stream_t stream);
+
 /*
  * ws_spgemm_wait -- synchronises `stream` and returns the device status
- * recorded by the last symbolic/numeric pass of C (WS_OK if none failed).
+ * recorded by the last symbolic/numeric pass of C (WS_OK if none failed);
+ * serves the elementwise passes too.
  */
 ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream);
 

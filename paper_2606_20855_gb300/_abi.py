@@ -43,7 +43,11 @@ SIGNATURES = [
     ("ws_spgemm_plan_info", _i32, [_p, ctypes.POINTER(_i64), _i32]),
     ("ws_set_tuning", _i32, [_i32, _i64]),
     ("ws_rowptr_scan_static", _i32, [_p, _i64, _p]),
+    ("ws_ewise_symbolic", _i32, [_p, _p, _p, _i32, ctypes.POINTER(_i64), _p]),
+    ("ws_ewise_numeric", _i32, [_p, _p, _p, _p, _p, _p]),
 ]
+
+EWISE_OPS = {"add": 1, "mul": 2}  # ws_ewise_op_t
 
 
 class WsError(RuntimeError):
@@ -100,6 +104,18 @@ def ws_spgemm_symbolic(A: int, B: int, C: int, stream: int) -> int:
 def ws_spgemm_numeric(A: int, B: int, C: int, c_colidx: int, c_vals: int, stream: int) -> None:
     _check("ws_spgemm_numeric", load().ws_spgemm_numeric(A, B, C, c_colidx or None, c_vals or None,
                                                          stream or None))
+
+
+def ws_ewise_symbolic(A: int, B: int, C: int, op, stream: int) -> int:
+    k = EWISE_OPS[op] if isinstance(op, str) else int(op)
+    nnz = ctypes.c_int64(-1)
+    _check("ws_ewise_symbolic", load().ws_ewise_symbolic(A, B, C, k, ctypes.byref(nnz), stream or None))
+    return nnz.value
+
+
+def ws_ewise_numeric(A: int, B: int, C: int, c_colidx: int, c_vals: int, stream: int) -> None:
+    _check("ws_ewise_numeric", load().ws_ewise_numeric(A, B, C, c_colidx or None, c_vals or None,
+                                                       stream or None))
 
 
 def ws_spgemm_wait(C: int, stream: int) -> None:

@@ -86,10 +86,21 @@ struct DevBuf {
   }
 };
 
+enum PlanKind { kPlanNone = 0, kPlanSpgemm = 1, kPlanEwise = 2 };
+
 struct Plan {
   DevBuf rows;    // per-row arrays + summary + scan partials
   DevBuf slices;  // dense-window slice arrays
   DevBuf ranks;   // register bitmap rows: kBmrSlots uint16 ranks per row of A
+  DevBuf ew;      // elementwise operations: summary, chunk arrays, scan partials
+  int kind = kPlanNone;  // which symbolic pass filled this plan
+  // elementwise plan (kPlanEwise)
+  int ew_op = 0, ew_group = 32;
+  int64_t ew_diag = 0, ew_nc_max = 0;
+  int64_t* ew_chunk_begin = nullptr;
+  int32_t* ew_chunk_row = nullptr;
+  int64_t* ew_chunk_off = nullptr;
+  int64_t* ew_partials = nullptr;
   DevSummary* host_sum = nullptr;  // pinned
   // carved pointers
   DevSummary* dsum = nullptr;
@@ -305,7 +316,9 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
   const int dev = C->device;
   const int sms = num_sms_of(dev);
   pl->ready = false;
+  pl->kind = kPlanSpgemm;
   pl->sym_launches = 0;
+  pl->num_launches = 0;
   pl->log2_group = log2_group_for(B);
   pl->run_limit = g_run_limit;
   pl->dense_width = g_dense_width > 0 ? g_dense_width : (sizeof(T) == 8 ? 8192 : 16384);
@@ -428,6 +441,114 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
   return WS_OK;
 }
 
+// ----------------------------------------------------- elementwise operations
+
+// Lanes per chunk from the mean merged row length (entries of A and B per row).
+int ewise_group_for(int64_t m, int64_t merged) {
+  const double avg = m > 0 ? static_cast<double>(merged) / static_cast<double>(m) : 0.0;
+  if (avg <= 8.0) return 4;
+  if (avg <= 16.0) return 8;
+  if (avg <= 32.0) return 16;
+  return 32;
+}
+
+ws_status_t carve_ewise(Plan* pl, int64_t m, int64_t nc_max, cudaStream_t s) {
+  const int64_t nb = scan_partials_needed(m > nc_max ? m : nc_max);
+  size_t off = 0;
+  const size_t o_sum = off; off = align_up(off + sizeof(DevSummary), 256);
+  const size_t o_begin = off; off = align_up(off + 8 * static_cast<size_t>(m + 1), 256);
+  const size_t o_row = off; off = align_up(off + 4 * static_cast<size_t>(nc_max), 256);
+  const size_t o_off = off; off = align_up(off + 8 * static_cast<size_t>(nc_max + 1), 256);
+  const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
+  ws_status_t st = pl->ew.reserve(off, s);
+  if (st != WS_OK) return st;
+  char* b = static_cast<char*>(pl->ew.ptr);
+  pl->dsum = reinterpret_cast<DevSummary*>(b + o_sum);
+  pl->ew_chunk_begin = reinterpret_cast<int64_t*>(b + o_begin);
+  pl->ew_chunk_row = reinterpret_cast<int32_t*>(b + o_row);
+  pl->ew_chunk_off = reinterpret_cast<int64_t*>(b + o_off);
+  pl->ew_partials = reinterpret_cast<int64_t*>(b + o_part);
+  return WS_OK;
+}
+
+template <typename T>
+EwisePlan<T> make_ewise(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, const Plan* pl) {
+  EwisePlan<T> p{};
+  p.A = {A->rowptr, A->colidx, static_cast<const T*>(A->vals)};
+  p.B = {B->rowptr, B->colidx, static_cast<const T*>(B->vals)};
+  p.m = A->nrows;
+  p.c_rowptr = C->rowptr;
+  p.c_colidx = C->colidx;
+  p.c_vals = static_cast<T*>(C->vals);
+  p.chunk_begin = pl->ew_chunk_begin;
+  p.chunk_row = pl->ew_chunk_row;
+  p.chunk_off = pl->ew_chunk_off;
+  p.nc_max = pl->ew_nc_max;
+  p.partials = pl->ew_partials;
+  p.sum = pl->dsum;
+  p.diag = pl->ew_diag;
+  p.group = pl->ew_group;
+  p.op = pl->ew_op;
+  return p;
+}
+
+template <typename T>
+ws_status_t ewise_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan* pl, int op,
+                                cudaStream_t s, int64_t* nnz_out) {
+  const int64_t m = A->nrows;
+  pl->ready = false;
+  pl->kind = kPlanEwise;
+  pl->sym_launches = 0;
+  pl->num_launches = 0;
+  pl->ew_op = op;
+  const int64_t merged = A->nnz + B->nnz;
+  pl->ew_group = ewise_group_for(m, merged);
+  pl->ew_diag = 16 * static_cast<int64_t>(pl->ew_group);
+  pl->ew_nc_max = m + merged / pl->ew_diag + 1;  // row i has at most 1 + len_i / diag chunks
+  ws_status_t st = carve_ewise(pl, m, pl->ew_nc_max, s);
+  if (st != WS_OK) return st;
+  WS_CUDA(cudaMemsetAsync(pl->dsum, 0, sizeof(DevSummary), s), "cudaMemsetAsync(summary)");
+  WS_CUDA(cudaMemsetAsync(C->rowptr, 0, sizeof(int64_t), s), "cudaMemsetAsync(rowptr[0])");
+  WS_CUDA(cudaMemsetAsync(pl->ew_chunk_begin, 0, sizeof(int64_t), s), "cudaMemsetAsync(chunk_begin[0])");
+  WS_CUDA(cudaMemsetAsync(pl->ew_chunk_off, 0, sizeof(int64_t), s), "cudaMemsetAsync(chunk_off[0])");
+  if (m > 0) {
+    launch_ewise_symbolic<T>(make_ewise<T>(A, B, C, pl), num_sms_of(C->device), s, &pl->sym_launches);
+    WS_CUDA(cudaGetLastError(), "elementwise symbolic launches");
+  }
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  st = device_status(*pl->host_sum);
+  if (st != WS_OK) return st;
+  C->nnz = m > 0 ? pl->host_sum->nnz : 0;
+  pl->products = merged;
+  pl->A = A;
+  pl->B = B;
+  pl->a_nnz = A->nnz;
+  pl->b_nnz = B->nnz;
+  pl->ready = true;
+  *nnz_out = C->nnz;
+  return WS_OK;
+}
+
+// Shared checks of the operand and output handles; creates C's plan.
+ws_status_t prepare_output(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C) {
+  if (C == A || C == B) return fail(WS_ERR_INVALID_ARG, "C must be a separate output handle");
+  if (A->dtype != B->dtype || C->dtype != A->dtype) return fail(WS_ERR_DTYPE, "A, B and C dtypes differ");
+  if (!C->plan) {
+    C->plan = new (std::nothrow) Plan;
+    if (!C->plan) return fail(WS_ERR_ALLOC, "host allocation failed");
+  }
+  Plan* pl = C->plan;
+  if (!pl->host_sum) {
+    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&pl->host_sum), sizeof(DevSummary));
+    if (e != cudaSuccess) {
+      pl->host_sum = nullptr;
+      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
+    }
+  }
+  return WS_OK;
+}
+
 ws_status_t check_handle(const ws_csr_s* h, const char* name) {
   if (!h) return fail(WS_ERR_INVALID_ARG, "%s is NULL", name);
   return WS_OK;
@@ -503,18 +624,8 @@ ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_
                 (long long)A->nrows, (long long)B->ncols);
   if (A->dtype != B->dtype || C->dtype != A->dtype) return fail(WS_ERR_DTYPE, "A, B and C dtypes differ");
   if (A->nnz > 0 && B->nrows == 0) return fail(WS_ERR_INVALID_CSR, "A has entries but B has no rows");
-  if (!C->plan) {
-    C->plan = new (std::nothrow) Plan;
-    if (!C->plan) return fail(WS_ERR_ALLOC, "host allocation failed");
-  }
+  if ((st = prepare_output(A, B, C)) != WS_OK) return st;
   Plan* pl = C->plan;
-  if (!pl->host_sum) {
-    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&pl->host_sum), sizeof(DevSummary));
-    if (e != cudaSuccess) {
-      pl->host_sum = nullptr;
-      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
-    }
-  }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   C->nnz = -1;
   if (A->dtype == WS_F64) return symbolic_impl<double>(A, B, C, pl, s, nnz_out);
@@ -529,7 +640,8 @@ ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_col
       (st = check_handle(C, "C")) != WS_OK)
     return st;
   Plan* pl = C->plan;
-  if (!pl || !pl->ready) return fail(WS_ERR_STATE, "numeric called before a successful symbolic pass");
+  if (!pl || !pl->ready || pl->kind != kPlanSpgemm)
+    return fail(WS_ERR_STATE, "numeric called before a successful SpGEMM symbolic pass");
   if (pl->A != A || pl->B != B || pl->a_nnz != A->nnz || pl->b_nnz != B->nnz)
     return fail(WS_ERR_STATE, "numeric called with other operands than the symbolic pass");
   if (C->nnz > 0 && (!c_colidx || !c_vals)) return fail(WS_ERR_INVALID_ARG, "c_colidx/c_vals NULL with nnz(C) > 0");
@@ -538,6 +650,56 @@ ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_col
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (A->dtype == WS_F64) return numeric_impl<double>(A, B, C, pl, s);
   return numeric_impl<float>(A, B, C, pl, s);
+}
+
+ws_status_t ws_ewise_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int op, int64_t* nnz_out, ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  if (!nnz_out) return fail(WS_ERR_INVALID_ARG, "nnz_out is NULL");
+  if (op != WS_EWISE_ADD && op != WS_EWISE_MUL) return fail(WS_ERR_INVALID_ARG, "unknown elementwise op %d", op);
+  if (A->nrows != B->nrows || A->ncols != B->ncols)
+    return fail(WS_ERR_SHAPE, "A is %lldx%lld but B is %lldx%lld", (long long)A->nrows, (long long)A->ncols,
+                (long long)B->nrows, (long long)B->ncols);
+  if (C->nrows != A->nrows || C->ncols != A->ncols)
+    return fail(WS_ERR_SHAPE, "C is %lldx%lld, expected %lldx%lld", (long long)C->nrows, (long long)C->ncols,
+                (long long)A->nrows, (long long)A->ncols);
+  if ((st = prepare_output(A, B, C)) != WS_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  C->nnz = -1;
+  const int kop = op == WS_EWISE_ADD ? kEwiseAdd : kEwiseMul;
+  if (A->dtype == WS_F64) return ewise_symbolic_impl<double>(A, B, C, C->plan, kop, s, nnz_out);
+  return ewise_symbolic_impl<float>(A, B, C, C->plan, kop, s, nnz_out);
+}
+
+ws_status_t ws_ewise_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                             ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  Plan* pl = C->plan;
+  if (!pl || !pl->ready || pl->kind != kPlanEwise)
+    return fail(WS_ERR_STATE, "numeric called before a successful elementwise symbolic pass");
+  if (pl->A != A || pl->B != B || pl->a_nnz != A->nnz || pl->b_nnz != B->nnz)
+    return fail(WS_ERR_STATE, "numeric called with other operands than the symbolic pass");
+  if (C->nnz > 0 && (!c_colidx || !c_vals)) return fail(WS_ERR_INVALID_ARG, "c_colidx/c_vals NULL with nnz(C) > 0");
+  C->colidx = c_colidx;
+  C->vals = c_vals;
+  pl->num_launches = 0;
+  if (C->nnz == 0) return WS_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int sms = num_sms_of(C->device);
+  if (A->dtype == WS_F64) {
+    launch_ewise_numeric<double>(make_ewise<double>(A, B, C, pl), sms, s, &pl->num_launches);
+  } else {
+    launch_ewise_numeric<float>(make_ewise<float>(A, B, C, pl), sms, s, &pl->num_launches);
+  }
+  WS_CUDA(cudaGetLastError(), "elementwise numeric launch");
+  return WS_OK;
 }
 
 ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
@@ -557,10 +719,11 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
 ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
-    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr) cudaDeviceSynchronize();
+    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr) cudaDeviceSynchronize();
     h->plan->rows.release();
     h->plan->slices.release();
     h->plan->ranks.release();
+    h->plan->ew.release();
     if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
     delete h->plan;
   }

@@ -148,6 +148,33 @@ struct RowPlan {
   int dense_width;     // dense-window slice width in columns
 };
 
+// Elementwise operations C = A op B on CSR matrices of one shape.
+constexpr int kEwiseAdd = 1;  // SpAdd: pattern union, values added
+constexpr int kEwiseMul = 2;  // Hadamard product: pattern intersection, values multiplied
+
+template <typename T>
+struct EwisePlan {
+  CsrView<T> A;
+  CsrView<T> B;
+  int64_t m;
+  int64_t* c_rowptr;
+  int32_t* c_colidx;     // numeric only
+  T* c_vals;             // numeric only
+  int64_t* chunk_begin;  // [m + 1]: first chunk of each row (chunks per row, then scanned in place)
+  int32_t* chunk_row;    // [nc_max]: row of each chunk
+  int64_t* chunk_off;    // [nc_max + 1]: C offset of each chunk (counts, then scanned in place)
+  int64_t nc_max;        // bound on the number of chunks: m + (nnz(A) + nnz(B)) / diag + 1
+  int64_t* partials;     // scan scratch for max(m, nc_max) entries
+  DevSummary* sum;
+  int64_t diag;          // merged positions per chunk
+  int group;             // lanes per chunk (4, 8, 16, 32)
+  int op;                // kEwiseAdd or kEwiseMul
+};
+template <typename T>
+void launch_ewise_symbolic(const EwisePlan<T>& p, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_ewise_numeric(const EwisePlan<T>& p, int num_sms, cudaStream_t s, int* launches);
+
 // Host-side launchers (one translation unit each).
 struct AnalyzeParams {
   int64_t m;

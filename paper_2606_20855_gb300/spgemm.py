@@ -134,6 +134,62 @@ class SpGEMM:
             pass
 
 
+class Ewise:
+    """A reusable elementwise operation C = A op B (op "add": SpAdd on the
+    union of the patterns; op "mul": Hadamard product on their intersection).
+
+    ``symbolic()`` returns nnz(C) (and synchronises the stream), ``numeric()``
+    queues the value pass and returns C as a :class:`DeviceCSR`.
+    """
+
+    def __init__(self, A: DeviceCSR, B: DeviceCSR, op: str = "add", validate: bool = False, stream=None):
+        if A.dtype != B.dtype:
+            raise TypeError("A and B must have the same value dtype")
+        if op not in _abi.EWISE_OPS:
+            raise ValueError(f"op must be one of {tuple(_abi.EWISE_OPS)}, got {op!r}")
+        self.A, self.B, self.op = A, B, op
+        s = _stream_handle(stream)
+        self._hA = self._hB = self._hC = None
+        self.device = A.rowptr.device
+        self._hA = A._handle(validate, s)
+        self._hB = B._handle(validate, s)
+        self.c_rowptr = torch.empty(A.nrows + 1, dtype=torch.int64, device=self.device)
+        self._hC = _abi.ws_csr_create(A.nrows, A.ncols, 0, self.c_rowptr.data_ptr(), 0, 0,
+                                      _DTYPES[A.dtype], False, s)
+        self.nnz = None
+
+    def symbolic(self, stream=None) -> int:
+        self.nnz = _abi.ws_ewise_symbolic(self._hA, self._hB, self._hC, self.op, _stream_handle(stream))
+        return self.nnz
+
+    def numeric(self, out: DeviceCSR | None = None, stream=None) -> DeviceCSR:
+        if self.nnz is None:
+            raise RuntimeError("symbolic() must run before numeric()")
+        if out is None or out.nnz != self.nnz:
+            colidx = torch.empty(self.nnz, dtype=torch.int32, device=self.device)
+            vals = torch.empty(self.nnz, dtype=self.A.dtype, device=self.device)
+            out = DeviceCSR(self.A.nrows, self.A.ncols, self.c_rowptr, colidx, vals)
+        _abi.ws_ewise_numeric(self._hA, self._hB, self._hC, out.colidx.data_ptr() if self.nnz else 0,
+                              out.vals.data_ptr() if self.nnz else 0, _stream_handle(stream))
+        return out
+
+    wait = SpGEMM.wait
+    plan_info = SpGEMM.plan_info
+    close = SpGEMM.close
+    __enter__ = SpGEMM.__enter__
+    __exit__ = SpGEMM.__exit__
+    __del__ = SpGEMM.__del__
+
+
+def ewise(A: DeviceCSR, B: DeviceCSR, op: str = "add", validate: bool = False, stream=None) -> DeviceCSR:
+    """C = A + B (op "add") or C = A .* B (op "mul") for CSR matrices of one shape on the GPU."""
+    with Ewise(A, B, op, validate=validate, stream=stream) as e:
+        e.symbolic(stream)
+        C = e.numeric(stream=stream)
+        e.wait(stream)
+    return C
+
+
 def spgemm(A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None) -> DeviceCSR:
     """C = A*B for CSR matrices on the GPU (sorted columns, structural zeros kept)."""
     with SpGEMM(A, B, validate=validate, stream=stream) as op:
