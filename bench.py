@@ -12,6 +12,10 @@ C once, at their stored widths).
 
 Extra keys: `e2e` (the same product through the public Python API from
 pinned host inputs to the host copy of C, copies inside the timed region),
+With an elementwise workload (``--workload ewise_* --op add|mul``) a step is
+one elementwise operation C = A + B or C = A .* B and the value is its
+effective bandwidth in GB/s of compulsory bytes.
+
 `roofline` (the whole product -- symbolic + numeric, the span the throughput
 target is set on -- against the measured copy bandwidth, with each pass's own
 figure under `passes`), `cpu_baseline` (the CPU oracle on a bounded row sample, on
@@ -38,9 +42,10 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-from synth import WORKLOADS, workload  # noqa: E402
+from synth import EWISE_WORKLOADS, WORKLOADS, ewise_workload, workload  # noqa: E402
 
 METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per config"
+EWISE_METRIC = "SpAdd / Hadamard effective HBM GB/s (compulsory bytes: read A and B, write C)"
 DEFAULT_WORKLOAD = "uniform_rect_1m"
 NOMINAL_HBM_GBS = 8000.0
 
@@ -227,8 +232,14 @@ def barrier(world: int, pg) -> None:
         pg.barrier()
 
 
+def is_ewise(args) -> bool:
+    return args.workload in EWISE_WORKLOADS
+
+
 def load_workload(args):
     """The named workload, optionally cut to the first --rows rows of A."""
+    if is_ewise(args):
+        return ewise_workload(args.workload)
     A, B = workload(args.workload)
     if args.rows and args.rows < A.nrows:
         from synth import row_subset
@@ -239,6 +250,9 @@ def load_workload(args):
 def run_reference(args, world, rank) -> None:
     """CPU oracle arm: each step computes a bounded row sample on the host cores."""
     if rank != 0:
+        return
+    if is_ewise(args):
+        run_reference_ewise(args)
         return
     from oracle import oracle_spgemm
     A, B = load_workload(args)
@@ -269,18 +283,55 @@ def run_reference(args, world, rank) -> None:
     print(json.dumps(line), flush=True)
 
 
+def ewise_bytes(A, B, nnz_c: int) -> int:
+    s = A.vals.dtype.itemsize
+    return csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz_c, s)
+
+
+def ewise_oracle_timed(A, B, op: str, steps: int) -> tuple[float, int]:
+    """Seconds per oracle run (the whole operation: the elementwise oracle is
+    vectorised numpy and finishes the full input in seconds) and nnz(C)."""
+    from oracle import oracle_ewise
+    times, nnz = [], 0
+    for _ in range(steps):
+        t0 = time.perf_counter()
+        nnz = oracle_ewise(A, B, op).nnz
+        times.append(time.perf_counter() - t0)
+    return statistics.mean(times), nnz
+
+
+def run_reference_ewise(args) -> None:
+    A, B = load_workload(args)
+    if args.warmup > 0:
+        ewise_oracle_timed(A, B, args.op, args.warmup)
+    dt, nnz = ewise_oracle_timed(A, B, args.op, max(args.steps, 1))
+    value = ewise_bytes(A, B, nnz) / dt / 1e9
+    sample = f"whole operation ({A.nnz} + {B.nnz} entries), numpy on one core"
+    line = {
+        "impl": "reference", "metric": EWISE_METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * dt, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "op": args.op, "description": EWISE_WORKLOADS[args.workload]},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_ours(args, world, rank, local, pg) -> None:
     import torch
     from paper_2606_20855_gb300 import _abi
-    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, Ewise, SpGEMM
 
     _abi.load()
     device = torch.device(f"cuda:{local}")
     torch.cuda.set_device(device)
     A, B = load_workload(args)
     same = B is A
-    ub = products_per_row(A, B)
+    ew = is_ewise(args)
+    ub = np.zeros(A.nrows, dtype=np.int64) if ew else products_per_row(A, B)
     products = int(ub.sum())
+    make_op = (lambda x, y: Ewise(x, y, args.op)) if ew else SpGEMM
     s = 8 if A.vals.dtype == np.float64 else 4
     stream = torch.cuda.current_stream(device)
 
@@ -289,7 +340,7 @@ def run_ours(args, world, rank, local, pg) -> None:
     l2 = torch.cuda.get_device_properties(device).L2_cache_size
     flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
 
-    op = SpGEMM(dA, dB)
+    op = make_op(dA, dB)
     out = None
 
     def step():
@@ -344,7 +395,7 @@ def run_ours(args, world, rank, local, pg) -> None:
         def e2e_step():
             tA = DeviceCSR(A.nrows, A.ncols, *[t.to(device, non_blocking=True) for t in hA])
             tB = tA if same else DeviceCSR(B.nrows, B.ncols, *[t.to(device, non_blocking=True) for t in hB])
-            with SpGEMM(tA, tB) as op2:
+            with make_op(tA, tB) as op2:
                 op2.symbolic()
                 C = op2.numeric()
                 h_rp.copy_(C.rowptr, non_blocking=True)
@@ -361,7 +412,8 @@ def run_ours(args, world, rank, local, pg) -> None:
         e2e_s = reduce_max(time.perf_counter() - t0, world, pg, device)
         h2d = sum(t.numel() * t.element_size() for t in hA) + (0 if same else sum(t.numel() * t.element_size() for t in hB))
         d2h = h_rp.numel() * 8 + h_col.numel() * 4 + h_val.numel() * h_val.element_size()
-        e2e = {"value": round(2.0 * products * args.e2e_steps * world / e2e_s / 1e9, 3), "unit": "GFLOP/s",
+        e2e_work = algo_bytes if ew else 2.0 * products
+        e2e = {"value": round(e2e_work * args.e2e_steps * world / e2e_s / 1e9, 3), "unit": "GB/s" if ew else "GFLOP/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
 
     op.close()
@@ -380,15 +432,20 @@ def run_ours(args, world, rank, local, pg) -> None:
         if table is NUMERIC_TRAFFIC and args.traffic is not None:
             return args.traffic
         return table.get(args.workload)
-    value = 2.0 * products * args.steps * world / total_s / 1e9
     eff_gbs = algo_bytes * args.steps * world / total_s / 1e9
+    value = eff_gbs if ew else 2.0 * products * args.steps * world / total_s / 1e9
     base = None
     if args.cpu_baseline_s > 0:
-        base = cpu_baseline(A, B, ub, args.cpu_baseline_s)
+        if ew:
+            dt, _ = ewise_oracle_timed(A, B, args.op, 1)
+            base = {"value": round(algo_bytes / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                    "sample": f"whole operation, {dt:.1f} s, numpy on one core"}
+        else:
+            base = cpu_baseline(A, B, ub, args.cpu_baseline_s)
     line = {
-        "metric": METRIC,
+        "metric": EWISE_METRIC if ew else METRIC,
         "value": round(value, 3),
-        "unit": "GFLOP/s",
+        "unit": "GB/s" if ew else "GFLOP/s",
         "n_gpus": world,
         "steps": args.steps,
         "warmup": args.warmup,
@@ -400,9 +457,10 @@ def run_ours(args, world, rank, local, pg) -> None:
         "data": "synthetic",
         "config": {
             "workload": args.workload if not args.rows else f"{args.workload}[:{A.nrows} rows]",
-            "description": WORKLOADS[args.workload],
+            "description": EWISE_WORKLOADS[args.workload] if ew else WORKLOADS[args.workload],
             "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_a": A.nnz, "nnz_b": B.nnz, "nnz_c": int(nnz),
-            "products": products, "l2": "flushed between timed steps (write of a buffer > L2)",
+            **({"op": args.op} if ew else {"products": products}),
+            "l2": "flushed between timed steps (write of a buffer > L2)",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
         },
         "effective_hbm_gbs": round(eff_gbs, 1),
@@ -411,14 +469,16 @@ def run_ours(args, world, rank, local, pg) -> None:
                       "numeric_median": round(statistics.median(num_ms), 4),
                       "step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
         "roofline": dict(roofline_obj(algo_bytes, statistics.mean(step_ms) / 1e3, peaks, traffic(None)),
-                         kernel="whole product: symbolic pass (nnz read-back included) + numeric pass",
+                         kernel=("whole operation" if ew else "whole product") +
+                                ": symbolic pass (nnz read-back included) + numeric pass",
                          passes={
                              "symbolic": dict(roofline_obj(sym_bytes, statistics.mean(sym_ms) / 1e3, peaks,
                                                            traffic(SYMBOLIC_TRAFFIC)),
                                               kernel="symbolic pass (compulsory bytes: structure of A and B "
                                                      "read once, C.rowptr written)"),
                              "numeric": dict(roofline_obj(algo_bytes, num_mean_s, peaks, traffic(NUMERIC_TRAFFIC)),
-                                             kernel=f"numeric pass: {numeric_kernels(info)}"),
+                                             kernel="numeric pass: " + ("ew_merge_kernel" if ew else
+                                                                            numeric_kernels(info))),
                          }),
         "gpu_launches": int(launches_per_step * args.steps),
         "plan": info,
@@ -435,7 +495,8 @@ def main(argv=None) -> int:
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=list(WORKLOADS), default=DEFAULT_WORKLOAD)
+    ap.add_argument("--workload", choices=list(WORKLOADS) + list(EWISE_WORKLOADS), default=DEFAULT_WORKLOAD)
+    ap.add_argument("--op", choices=["add", "mul"], default="add", help="elementwise workloads: C = A + B or A .* B")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
     ap.add_argument("--ref-step-s", type=float, default=2.0, help="seconds per reference-arm step")

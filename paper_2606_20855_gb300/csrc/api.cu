@@ -33,6 +33,8 @@ int g_rcd_max_a = kRcdDefaultMaxA;
 int64_t g_wb_span = kWbMaxSpan;
 int g_run_limit = 64;
 int g_dense_width = 0;  // 0 = default per value type
+int g_ewise_lanes = 1;  // elementwise: lanes per chunk (0 = from the mean row length)
+int64_t g_ewise_diag = 64;  // elementwise, one thread per chunk: merged positions per chunk
 constexpr int kLongRowThreshold = 128;
 
 ws_status_t fail(ws_status_t st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
@@ -502,8 +504,8 @@ ws_status_t ewise_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* 
   pl->num_launches = 0;
   pl->ew_op = op;
   const int64_t merged = A->nnz + B->nnz;
-  pl->ew_group = ewise_group_for(m, merged);
-  pl->ew_diag = 16 * static_cast<int64_t>(pl->ew_group);
+  pl->ew_group = g_ewise_lanes > 0 ? g_ewise_lanes : ewise_group_for(m, merged);
+  pl->ew_diag = pl->ew_group == 1 ? g_ewise_diag : 16 * static_cast<int64_t>(pl->ew_group);
   pl->ew_nc_max = m + merged / pl->ew_diag + 1;  // row i has at most 1 + len_i / diag chunks
   ws_status_t st = carve_ewise(pl, m, pl->ew_nc_max, s);
   if (st != WS_OK) return st;
@@ -812,6 +814,15 @@ ws_status_t ws_set_tuning(int key, int64_t value) {
     case 7:
       if (value < 0 || value > kWbMaxSpan) return fail(WS_ERR_INVALID_ARG, "wide-bitmap span out of range");
       g_wb_span = value;
+      return WS_OK;
+    case 8:
+      if (value != 0 && value != 1 && value != 4 && value != 8 && value != 16 && value != 32)
+        return fail(WS_ERR_INVALID_ARG, "elementwise lanes per chunk must be 0, 1, 4, 8, 16 or 32");
+      g_ewise_lanes = static_cast<int>(value);
+      return WS_OK;
+    case 9:
+      if (value < 2 || value > (int64_t{1} << 20)) return fail(WS_ERR_INVALID_ARG, "elementwise chunk length out of range");
+      g_ewise_diag = value;
       return WS_OK;
   }
   return fail(WS_ERR_INVALID_ARG, "unknown tuning key %d", key);

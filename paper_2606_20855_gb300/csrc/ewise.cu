@@ -8,8 +8,7 @@
 //
 // Work units.  Row i is seen as the merge of its two sorted column lists
 // (length na_i + nb_i) and cut into chunks of `diag` merged positions
-// (merge-path diagonals; at least one chunk per row, so an empty row has one
-// empty chunk).  A chunk boundary is placed by a binary search on the two
+// (merge-path diagonals; an empty row has none).  A chunk boundary is placed by a binary search on the two
 // lists, with the entry of A ahead of an equal entry of B and an equal pair
 // never cut apart, so every chunk is the merge of a contiguous part of each
 // list and no position of C is produced by two chunks.  Chunks balance long
@@ -27,7 +26,7 @@
 //
 // Symbolic pass: chunks per row -> scan -> chunk -> row map -> count per
 // chunk -> scan (chunk output offsets, nnz(C)) -> C.rowptr[i] = offset of the
-// first chunk of row i.  Numeric pass: every chunk merges again and writes its
+// first chunk of row i (of the next chunk for an empty row).  Numeric pass: every chunk merges again and writes its
 // entries from its offset.
 #include <climits>
 
@@ -90,19 +89,27 @@ __device__ int64_t merge_chunk(const int32_t* a, const T* va, int64_t na, const 
     }
     const int limit = min(__shfl_sync(gmask, ca, G - 1, G), __shfl_sync(gmask, cb, G - 1, G));
     // la = #{b window < ca}, lb = #{a window < cb}
+    // Counting needs only the equal pairs (found from the A side); writing a
+    // union also needs the place of every B entry among the A entries.
+    constexpr bool kBSide = FILL && OP == kEwiseAdd;
     int la = 0, lb = 0;
 #pragma unroll
     for (int s = G / 2; s > 0; s >>= 1) {
       if (__shfl_sync(gmask, cb, la + s - 1, G) < ca) la += s;
-      if (__shfl_sync(gmask, ca, lb + s - 1, G) < cb) lb += s;
+      if constexpr (kBSide) {
+        if (__shfl_sync(gmask, ca, lb + s - 1, G) < cb) lb += s;
+      }
     }
     if (__shfl_sync(gmask, cb, la, G) < ca) ++la;
-    if (__shfl_sync(gmask, ca, lb, G) < cb) ++lb;
-    // every lane of the group takes part in each shuffle, so both run before the tests
+    // every lane of the group takes part in each shuffle, so they run before the tests
     const int cb_at = __shfl_sync(gmask, cb, la & (G - 1), G);
-    const int ca_at = __shfl_sync(gmask, ca, lb & (G - 1), G);
     const bool a_eq = la < G && cb_at == ca && ca != INT_MAX;
-    const bool b_eq = lb < G && ca_at == cb && cb != INT_MAX;
+    bool b_eq = false;
+    if constexpr (kBSide) {
+      if (__shfl_sync(gmask, ca, lb, G) < cb) ++lb;
+      const int ca_at = __shfl_sync(gmask, ca, lb & (G - 1), G);
+      b_eq = lb < G && ca_at == cb && cb != INT_MAX;
+    }
     T xb_at = T(0);
     if constexpr (FILL) xb_at = __shfl_sync(gmask, xb, la & (G - 1), G);
     const bool a_take = ca != INT_MAX && ca <= limit;
@@ -110,26 +117,27 @@ __device__ int64_t merge_chunk(const int32_t* a, const T* va, int64_t na, const 
     const unsigned ma = group_bits<G>(__ballot_sync(gmask, a_take), g);
     const unsigned mb = group_bits<G>(__ballot_sync(gmask, b_take), g);
     const unsigned below = below_mask(gl);
-    if constexpr (OP == kEwiseAdd) {
+    if constexpr (OP == kEwiseAdd && !FILL) {
+      // union size: every A and B entry taken, less one per equal pair
+      out += __popc(ma) + __popc(mb) - __popc(group_bits<G>(__ballot_sync(gmask, a_take && a_eq), g));
+    } else if constexpr (OP == kEwiseAdd) {
       const unsigned mbu = group_bits<G>(__ballot_sync(gmask, b_take && !b_eq), g);  // B-only entries
-      if constexpr (FILL) {
-        if (a_take) {
-          const int64_t q = out + gl + __popc(mbu & below_mask(la));
-          if (q < cap) {
-            out_c[q] = ca;
-            out_v[q] = a_eq ? xa + xb_at : xa;
-          } else {
-            *bad = true;
-          }
+      if (a_take) {
+        const int64_t q = out + gl + __popc(mbu & below_mask(la));
+        if (q < cap) {
+          out_c[q] = ca;
+          out_v[q] = a_eq ? xa + xb_at : xa;
+        } else {
+          *bad = true;
         }
-        if (b_take && !b_eq) {
-          const int64_t q = out + lb + __popc(mbu & below);
-          if (q < cap) {
-            out_c[q] = cb;
-            out_v[q] = xb;
-          } else {
-            *bad = true;
-          }
+      }
+      if (b_take && !b_eq) {
+        const int64_t q = out + lb + __popc(mbu & below);
+        if (q < cap) {
+          out_c[q] = cb;
+          out_v[q] = xb;
+        } else {
+          *bad = true;
         }
       }
       out += __popc(ma) + __popc(mbu);
@@ -155,13 +163,140 @@ __device__ int64_t merge_chunk(const int32_t* a, const T* va, int64_t na, const 
   return out;
 }
 
+// Output writer of one thread: entries go out four at a time as 16-byte
+// stores once the position is a multiple of four (vec), singly before that
+// and for the last partial group.  Positions past `cap` are dropped and
+// flagged.
+template <typename T>
+struct SeqWriter {
+  int32_t* c;
+  T* v;
+  int64_t cap, n = 0, head = 0;
+  bool vec;
+  int bc0 = 0, bc1 = 0, bc2 = 0, bc3 = 0;
+  T bv0 = T(0), bv1 = T(0), bv2 = T(0), bv3 = T(0);
+
+  __device__ SeqWriter(int32_t* c_, T* v_, int64_t cap_, int64_t abs0, bool vec_) : c(c_), v(v_), cap(cap_), vec(vec_) {
+    head = vec ? ((4 - (abs0 & 3)) & 3) : cap;  // entries before the first 16-byte boundary
+  }
+  __device__ void put(int col, T val, bool* bad) {
+    if (n >= cap) {
+      *bad = true;
+      return;
+    }
+    if (n < head) {
+      c[n] = col;
+      v[n] = val;
+    } else {
+      const int slot = static_cast<int>((n - head) & 3);
+      bc0 = slot == 0 ? col : bc0;
+      bc1 = slot == 1 ? col : bc1;
+      bc2 = slot == 2 ? col : bc2;
+      bc3 = slot == 3 ? col : bc3;
+      bv0 = slot == 0 ? val : bv0;
+      bv1 = slot == 1 ? val : bv1;
+      bv2 = slot == 2 ? val : bv2;
+      bv3 = slot == 3 ? val : bv3;
+      if (slot == 3) {
+        const int64_t q = n - 3;
+        *reinterpret_cast<int4*>(c + q) = make_int4(bc0, bc1, bc2, bc3);
+        if constexpr (sizeof(T) == 4) {
+          *reinterpret_cast<float4*>(v + q) = make_float4(bv0, bv1, bv2, bv3);
+        } else {
+          reinterpret_cast<double2*>(v + q)[0] = make_double2(bv0, bv1);
+          reinterpret_cast<double2*>(v + q)[1] = make_double2(bv2, bv3);
+        }
+      }
+    }
+    ++n;
+  }
+  __device__ void flush() {
+    if (n <= head) return;
+    const int rest = static_cast<int>((n - head) & 3);
+    const int64_t q = n - rest;
+    if (rest > 0) { c[q] = bc0; v[q] = bv0; }
+    if (rest > 1) { c[q + 1] = bc1; v[q + 1] = bv1; }
+    if (rest > 2) { c[q + 2] = bc2; v[q + 2] = bv2; }
+  }
+};
+
+// One thread merges a[0..na) with b[0..nb) entry by entry (the two lists sit
+// in a few cache lines each, so the loads after the first hit L1); returns
+// the number of outputs.  FILL: writes them through `w`.
+template <typename T, int OP, bool FILL>
+__device__ int64_t merge_seq(const int32_t* a, const T* va, int64_t na, const int32_t* b, const T* vb, int64_t nb,
+                             SeqWriter<T>* w, bool* bad) {
+  int64_t i = 0, j = 0, out = 0;
+  int ca = na > 0 ? a[0] : INT_MAX;
+  int cb = nb > 0 ? b[0] : INT_MAX;
+  for (int64_t step = 0; step < na + nb && (i < na || j < nb); ++step) {
+    const bool take_a = ca <= cb, take_b = cb <= ca;
+    if constexpr (OP == kEwiseAdd) {
+      if constexpr (FILL) w->put(take_a ? ca : cb, take_a && take_b ? va[i] + vb[j] : (take_a ? va[i] : vb[j]), bad);
+      ++out;
+    } else if (take_a && take_b) {
+      if constexpr (FILL) w->put(ca, va[i] * vb[j], bad);
+      ++out;
+    }
+    if (take_a) {
+      ++i;
+      ca = i < na ? a[i] : INT_MAX;
+    }
+    if (take_b) {
+      ++j;
+      cb = j < nb ? b[j] : INT_MAX;
+    }
+  }
+  if (i < na || j < nb) *bad = true;  // only for unsorted input: the step bound ran out
+  if constexpr (FILL) w->flush();
+  return out;
+}
+
+// One thread per chunk, same contract as ew_merge_kernel.
+template <typename T, int OP, bool FILL>
+__global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(const EwisePlan<T> p) {
+  const int64_t nc = p.chunk_begin[p.m];
+  bool bad = false;
+  // 16-byte stores need 16-byte aligned C arrays (any allocation is)
+  const bool vec = ((reinterpret_cast<uintptr_t>(p.c_colidx) | reinterpret_cast<uintptr_t>(p.c_vals)) & 15u) == 0;
+  for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < p.nc_max;
+       c += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    if (c >= nc) {
+      if (!FILL) p.chunk_off[c + 1] = 0;
+      continue;
+    }
+    const int32_t row = p.chunk_row[c];
+    const int64_t k = c - p.chunk_begin[row];
+    const int64_t a0 = p.A.rowptr[row], na = p.A.rowptr[row + 1] - a0;
+    const int64_t b0 = p.B.rowptr[row], nb = p.B.rowptr[row + 1] - b0;
+    const int32_t* a = p.A.colidx + a0;
+    const int32_t* b = p.B.colidx + b0;
+    const int64_t d0 = k * p.diag;
+    const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
+    int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
+    if (d0 > 0) merge_split(a, na, b, nb, d0, &i0, &j0);
+    if (d1 < na + nb) merge_split(a, na, b, nb, d1, &i1, &j1);
+    if constexpr (FILL) {
+      const int64_t o0 = p.chunk_off[c];
+      const int64_t cap = p.chunk_off[c + 1] - o0;
+      SeqWriter<T> w(p.c_colidx + o0, p.c_vals + o0, cap, o0, vec);
+      const int64_t n = merge_seq<T, OP, true>(a + i0, p.A.vals + a0 + i0, i1 - i0, b + j0, p.B.vals + b0 + j0,
+                                               j1 - j0, &w, &bad);
+      if (n != cap) bad = true;
+    } else {
+      p.chunk_off[c + 1] = merge_seq<T, OP, false>(a + i0, nullptr, i1 - i0, b + j0, nullptr, j1 - j0, nullptr, &bad);
+    }
+  }
+  if (bad) atomicOr(&p.sum->status, kErrCount);
+}
+
 __global__ void __launch_bounds__(kEwThreads) ew_chunks_per_row_kernel(int64_t m, const int64_t* arp,
                                                                        const int64_t* brp, int64_t diag,
                                                                        int64_t* chunk_begin) {
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < m;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int64_t len = (arp[i + 1] - arp[i]) + (brp[i + 1] - brp[i]);
-    chunk_begin[i + 1] = len > diag ? (len + diag - 1) / diag : 1;
+    chunk_begin[i + 1] = (len + diag - 1) / diag;  // an empty row has no chunk
   }
 }
 
@@ -178,7 +313,7 @@ __global__ void __launch_bounds__(kEwThreads) ew_chunk_rows_kernel(int64_t m, co
 // chunk c (0 for c beyond the last chunk).  FILL: writes chunk c's outputs
 // from C offset chunk_off[c].
 template <typename T, int G, int OP, bool FILL>
-__global__ void __launch_bounds__(kEwThreads) ew_merge_kernel(const EwisePlan<T> p) {
+__global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_kernel(const EwisePlan<T> p) {
   constexpr int kGroups = 32 / G;
   const int lane = threadIdx.x & 31;
   const int g = lane / G, gl = lane % G;
@@ -241,6 +376,10 @@ void launch_merge(const EwisePlan<T>& p, int num_sms, cudaStream_t s) {
 
 template <typename T, int OP, bool FILL>
 void launch_merge_g(const EwisePlan<T>& p, int num_sms, cudaStream_t s) {
+  if (p.group == 1) {
+    ew_merge_seq_kernel<T, OP, FILL><<<grid_for(p.nc_max, kEwThreads, num_sms, 8), kEwThreads, 0, s>>>(p);
+    return;
+  }
   switch (p.group) {
     case 4: launch_merge<T, 4, OP, FILL>(p, num_sms, s); break;
     case 8: launch_merge<T, 8, OP, FILL>(p, num_sms, s); break;

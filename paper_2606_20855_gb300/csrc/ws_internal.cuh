@@ -167,7 +167,7 @@ struct EwisePlan {
   int64_t* partials;     // scan scratch for max(m, nc_max) entries
   DevSummary* sum;
   int64_t diag;          // merged positions per chunk
-  int group;             // lanes per chunk (4, 8, 16, 32)
+  int group;             // lanes per chunk (1: one thread merges entry by entry; 4, 8, 16, 32: windows)
   int op;                // kEwiseAdd or kEwiseMul
 };
 template <typename T>

@@ -19,7 +19,7 @@ from oracle import oracle_ewise
 from paper_2606_20855_gb300 import _abi
 from paper_2606_20855_gb300.spgemm import DeviceCSR, Ewise, SpGEMM
 from synth import EWISE_WORKLOADS, HostCSR, ewise_workload, random_csr, uniform_csr
-from tests._gpu import device_invariants
+from tests._gpu import device_invariants, tuning
 from tests._helpers import TOL, check_csr_invariants, value_error
 
 pytestmark = pytest.mark.gpu
@@ -53,27 +53,37 @@ def check(A, B, op, validate=False):
     return info
 
 
+# lanes per chunk: 1 (one thread per chunk, the default) and 0 (lane groups
+# of 4..32 sized from the mean row length)
+LANES = [1, 0]
+
+
+@pytest.mark.parametrize("lanes", LANES)
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("dtype", DTYPES)
 @pytest.mark.parametrize("seed", range(10))
-def test_random_shapes(seed, dtype, op):
+def test_random_shapes(seed, dtype, op, lanes):
     rng = np.random.default_rng(900 + seed)
     m, n = (int(x) for x in rng.integers(1, 500, size=2))
     A = random_csr(m, n, float(rng.choice([0.005, 0.03, 0.2])), rng, dtype, "sym", empty_rows=0.1)
     B = random_csr(m, n, float(rng.choice([0.005, 0.03, 0.2])), rng, dtype, "sym", empty_rows=0.1)
-    check(A, B, op, validate=True)
+    with tuning(ewise_lanes=lanes):
+        check(A, B, op, validate=True)
 
 
+@pytest.mark.parametrize("lanes", LANES)
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("per_row", [2, 6, 12, 40, 200])
-def test_every_group_size(per_row, op):
-    # mean merged row lengths 4 .. 400 select 4, 8, 16 and 32 lanes per chunk;
-    # 30,011 rows give many CTAs and a ragged last one
+def test_every_group_size(per_row, op, lanes):
+    # mean merged row lengths 4 .. 400 select 4, 8, 16 and 32 lanes per chunk
+    # (lanes 0), or cut rows into 1..7 chunks of 64 (lanes 1); 30,011 rows
+    # give many CTAs and a ragged last one
     rng = np.random.default_rng(per_row)
     n = max(64, per_row * per_row // 2)  # rejection sampling of distinct columns needs n >> per_row^2 / 2
     A = uniform_csr(30_011, n, per_row, rng, np.float64, "sym")
     B = uniform_csr(30_011, n, per_row, rng, np.float64, "sym")
-    check(A, B, op)
+    with tuning(ewise_lanes=lanes):
+        check(A, B, op)
 
 
 def _long_rows(m, n, lens, rng, overlap):
@@ -93,15 +103,18 @@ def _long_rows(m, n, lens, rng, overlap):
     return build(ra), build(rb)
 
 
+@pytest.mark.parametrize("lanes,chunk", [(1, 64), (1, 2), (1, 7), (0, 64), (32, 64)])
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("overlap", [0.0, 0.5, 1.0])
-def test_long_rows_many_chunks(overlap, op):
-    # rows of up to 20,000 entries per operand are cut into hundreds of chunks;
-    # with overlap 1.0 every column is an equal pair, so pairs meet every cut
+def test_long_rows_many_chunks(overlap, op, lanes, chunk):
+    # rows of up to 20,000 entries per operand are cut into hundreds of chunks
+    # (tens of thousands with chunks of 2); with overlap 1.0 every column is an
+    # equal pair, so pairs meet every cut
     rng = np.random.default_rng(31)
     lens = [20_000, 1, 0, 5_000, 777, 3, 12_345, 64, 65, 0]
     A, B = _long_rows(len(lens), 40_000, lens, rng, overlap)
-    check(A, B, op)
+    with tuning(ewise_lanes=lanes, ewise_chunk=chunk):
+        check(A, B, op)
 
 
 @pytest.mark.parametrize("op", OPS)
