@@ -9,7 +9,8 @@ C (all rows when ``rows`` is None) as numpy arrays computed by
 ``spgemm_oracle.cpp`` (Gustavson's row-wise algorithm with an ordered map per
 row, Sec. 5.1), with values accumulated in float64, plus
 absmass = sum |a*b| per output entry.  ``oracle_ewise(A, B, op)`` (ewise.py)
-is the elementwise SpAdd / Hadamard oracle.
+is the elementwise SpAdd / Hadamard oracle, ``oracle_spmspv(A, x_idx, x_vals)``
+(spmspv.py) the sparse matrix - sparse vector product.
 """
 from __future__ import annotations
 
@@ -101,5 +102,6 @@ def oracle_spgemm(A, B, rows=None, threads: int = 1) -> OracleCSR:
 
 
 from .ewise import oracle_ewise  # noqa: E402  (needs OracleCSR above)
+from .spmspv import OracleSparseVector, oracle_spmspv  # noqa: E402
 
-__all__ = ["oracle_spgemm", "oracle_ewise", "OracleCSR", "build", "LIB"]
+__all__ = ["oracle_spgemm", "oracle_ewise", "oracle_spmspv", "OracleCSR", "OracleSparseVector", "build", "LIB"]

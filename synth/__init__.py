@@ -3,5 +3,6 @@
 Holds input generation only; no part of the sparse product is computed here.
 """
 from .matrices import *  # noqa: F401,F403
-from .matrices import (EWISE_WORKLOADS, HostCSR, WORKLOADS, WORKLOAD_ORDER, ewise_workload,  # noqa: F401
-                       permute_symmetric, row_subset, workload)
+from .matrices import (EWISE_WORKLOADS, SPMSPV_WORKLOADS, HostCSR, WORKLOADS, WORKLOAD_ORDER,  # noqa: F401
+                       ewise_workload, permute_symmetric, row_subset, sparse_vector, spmspv_workload,
+                       transpose_csr, workload)

@@ -47,6 +47,10 @@ __all__ = [
     "permute_symmetric",
     "ewise_workload",
     "EWISE_WORKLOADS",
+    "transpose_csr",
+    "sparse_vector",
+    "spmspv_workload",
+    "SPMSPV_WORKLOADS",
 ]
 
 
@@ -274,6 +278,45 @@ def ewise_workload(name: str):
     if name == "ewise_rmat20_same":
         return A, A
     return A, permute_symmetric(A, rng.permutation(A.nrows))
+
+
+def transpose_csr(A: HostCSR) -> HostCSR:
+    """A^T in CSR (= A in CSC): row j lists the rows i of A's entries in column j, ascending."""
+    rows = np.repeat(np.arange(A.nrows, dtype=np.int64), np.diff(A.rowptr))
+    cols = A.colidx.astype(np.int64)
+    order = np.argsort(cols * max(A.nrows, 1) + rows, kind="stable")
+    rowptr = np.zeros(A.ncols + 1, dtype=np.int64)
+    np.cumsum(np.bincount(cols, minlength=A.ncols), out=rowptr[1:])
+    return HostCSR(A.ncols, A.nrows, rowptr, rows[order].astype(np.int32), A.vals[order])
+
+
+def sparse_vector(n: int, density: float, rng: np.random.Generator, dtype=np.float64,
+                  kind: str = "pos") -> tuple[np.ndarray, np.ndarray]:
+    """A sparse vector of length n: round(density * n) distinct indices drawn
+    uniformly without replacement (sorted, int32) and values (see _draw_values)."""
+    k = int(round(density * n))
+    idx = np.sort(rng.choice(n, size=k, replace=False)).astype(np.int32) if k else np.zeros(0, np.int32)
+    return idx, _draw_values(rng, k, kind).astype(dtype)
+
+
+# Inputs of the sparse matrix - sparse vector product y = A x: a power-law
+# graph standing in for the SNAP matrices of the paper's SpMSpV benchmark,
+# and a vector with 90% of its entries zero.
+SPMSPV_WORKLOADS = {
+    "spmspv_rmat20": "R-MAT 2^20, edge factor 16, (a,b,c,d)=(.57,.19,.19,.05), fp64 values in (0,1], seed 5; "
+                     "x: 10% of the 2^20 indices drawn uniformly without replacement, values in (0,1]",
+}
+
+
+def spmspv_workload(name: str):
+    """Return (A, x_idx, x_vals) for a named SpMSpV workload."""
+    if name not in SPMSPV_WORKLOADS:
+        raise KeyError(f"unknown SpMSpV workload {name!r}; known: {list(SPMSPV_WORKLOADS)}")
+    rng = np.random.default_rng(5)
+    rp, ci, _ = rmat_pattern(20, 16, RMAT_PROBS, rng)
+    A = HostCSR(1 << 20, 1 << 20, rp, ci, _draw_values(rng, ci.size, "pos").astype(np.float64))
+    x_idx, x_vals = sparse_vector(A.ncols, 0.1, rng, np.float64, "pos")
+    return A, x_idx, x_vals
 
 
 def row_subset(A: HostCSR, rows: np.ndarray) -> HostCSR:
