@@ -163,6 +163,32 @@ ws_status_t ws_ewise_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_coli
                              ws_stream_t stream);
 
 /*
+ * ws_spmspv -- sparse matrix - sparse vector product y = A x (Sec. 5.2,
+ * "Sparse Linear Algebra": SpMSpV, where x's stored entries select columns of
+ * A and the columns are accumulated into a sparse byte-map over y that a
+ * merge level protects).
+ *   At      handle of A^T in CSR, i.e. A by columns: At is n x m for an m x n
+ *           A, and row j of At lists the rows i of A's entries in column j
+ *           (ascending) with their values
+ *   nnz_x   stored entries of x, 0 <= nnz_x <= n
+ *   x_idx   device int32[nnz_x], strictly increasing, in [0, n)
+ *   x_vals  device values [nnz_x] of At's dtype
+ *   y_idx   device int32[m] (capacity m): receives y's indices, increasing
+ *   y_vals  device values [m] of At's dtype: receives y's values
+ *   nnz_y   host pointer: receives the number of stored entries of y
+ * y holds i iff some stored A[i,j] has j stored in x (structural: a sum of
+ * exactly 0.0 is kept), y[i] = sum of A[i,j] x[j] accumulated in the value
+ * type in unspecified order.  Work is queued on `stream` and the call
+ * synchronises it (to return nnz_y).  Device scratch (an accumulator and a
+ * bitmap of length m, offsets per x entry) is allocated stream-ordered and
+ * cached in At's handle.  Errors: WS_ERR_INVALID_ARG (NULL pointers, nnz_x out
+ * of range), WS_ERR_DEVICE (an index of x or of At out of range: those entries
+ * are skipped and flagged).
+ */
+ws_status_t ws_spmspv(ws_csr_t At, int64_t nnz_x, const int32_t* x_idx, const void* x_vals, int32_t* y_idx,
+                      void* y_vals, int64_t* nnz_y, ws_stream_t stream);
+
+/*
  * ws_spgemm_wait -- synchronises `stream` and returns the device status
  * recorded by the last symbolic/numeric pass of C (WS_OK if none failed);
  * serves the elementwise passes too.

@@ -1,5 +1,6 @@
 """GB300 (sm_103a) SpGEMM: C = A*B for CSR matrices, computed by hand-written CUDA kernels;
-also the elementwise operations C = A + B and C = A .* B.
+also the elementwise operations C = A + B and C = A .* B and the sparse
+matrix - sparse vector product y = A x.
 
 The C ABI lives in include/ws_spgemm.h and libws_spgemm.so (built by
 ``paper_2606_20855_gb300.build``).  ``_abi`` is the ctypes binding with the
@@ -7,7 +8,7 @@ same function names; ``spgemm`` holds the PyTorch-facing wrapper.  Importing
 this package loads nothing; the library is loaded on first use.
 """
 
-__all__ = ["DeviceCSR", "SpGEMM", "spgemm", "Ewise", "ewise"]
+__all__ = ["DeviceCSR", "SpGEMM", "spgemm", "Ewise", "ewise", "SpMSpV", "spmspv"]
 
 
 def __getattr__(name):

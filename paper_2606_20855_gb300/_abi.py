@@ -45,6 +45,7 @@ SIGNATURES = [
     ("ws_rowptr_scan_static", _i32, [_p, _i64, _p]),
     ("ws_ewise_symbolic", _i32, [_p, _p, _p, _i32, ctypes.POINTER(_i64), _p]),
     ("ws_ewise_numeric", _i32, [_p, _p, _p, _p, _p, _p]),
+    ("ws_spmspv", _i32, [_p, _i64, _p, _p, _p, _p, ctypes.POINTER(_i64), _p]),
 ]
 
 EWISE_OPS = {"add": 1, "mul": 2}  # ws_ewise_op_t
@@ -116,6 +117,13 @@ def ws_ewise_symbolic(A: int, B: int, C: int, op, stream: int) -> int:
 def ws_ewise_numeric(A: int, B: int, C: int, c_colidx: int, c_vals: int, stream: int) -> None:
     _check("ws_ewise_numeric", load().ws_ewise_numeric(A, B, C, c_colidx or None, c_vals or None,
                                                        stream or None))
+
+
+def ws_spmspv(At: int, nnz_x: int, x_idx: int, x_vals: int, y_idx: int, y_vals: int, stream: int) -> int:
+    nnz = ctypes.c_int64(-1)
+    _check("ws_spmspv", load().ws_spmspv(At, nnz_x, x_idx or None, x_vals or None, y_idx or None, y_vals or None,
+                                         ctypes.byref(nnz), stream or None))
+    return nnz.value
 
 
 def ws_spgemm_wait(C: int, stream: int) -> None:

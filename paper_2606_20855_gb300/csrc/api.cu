@@ -95,6 +95,7 @@ struct Plan {
   DevBuf slices;  // dense-window slice arrays
   DevBuf ranks;   // register bitmap rows: kBmrSlots uint16 ranks per row of A
   DevBuf ew;      // elementwise operations: summary, chunk arrays, scan partials
+  DevBuf sv;      // sparse matrix - sparse vector product (in A^T's handle): accumulator, bitmap, offsets
   int kind = kPlanNone;  // which symbolic pass filled this plan
   // elementwise plan (kPlanEwise)
   int ew_op = 0, ew_group = 32;
@@ -532,6 +533,80 @@ ws_status_t ewise_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* 
   return WS_OK;
 }
 
+// ------------------------------------------ sparse matrix - sparse vector
+
+// Creates a handle's plan and its pinned summary if missing.
+ws_status_t ensure_plan(ws_csr_s* h) {
+  if (!h->plan) {
+    h->plan = new (std::nothrow) Plan;
+    if (!h->plan) return fail(WS_ERR_ALLOC, "host allocation failed");
+  }
+  if (!h->plan->host_sum) {
+    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&h->plan->host_sum), sizeof(DevSummary));
+    if (e != cudaSuccess) {
+      h->plan->host_sum = nullptr;
+      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
+    }
+  }
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t spmspv_impl(ws_csr_s* At, int64_t nx, const int32_t* x_idx, const void* x_vals, int32_t* y_idx,
+                        void* y_vals, int64_t* nnz_y, cudaStream_t s) {
+  Plan* pl = At->plan;
+  const int64_t m = At->ncols, n = At->nrows;
+  const int64_t tiles = spmspv_tiles(m);
+  const int64_t words = (m + 31) / 32;
+  const int64_t nb = scan_partials_needed(nx > tiles ? nx : tiles);
+  size_t off = 0;
+  const size_t o_sum = off; off = align_up(off + sizeof(DevSummary), 256);
+  const size_t o_acc = off; off = align_up(off + sizeof(T) * static_cast<size_t>(m), 256);
+  const size_t o_bits = off; off = align_up(off + 4 * static_cast<size_t>(words), 256);
+  const size_t o_off = off; off = align_up(off + 8 * static_cast<size_t>(nx + 1), 256);
+  const size_t o_first = off; off = align_up(off + 8 * static_cast<size_t>(nx), 256);
+  const size_t o_cnt = off; off = align_up(off + 8 * static_cast<size_t>(tiles + 1), 256);
+  const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
+  ws_status_t st = pl->sv.reserve(off, s);
+  if (st != WS_OK) return st;
+  char* b = static_cast<char*>(pl->sv.ptr);
+  SpmspvPlan<T> p{};
+  p.At = {At->rowptr, At->colidx, static_cast<const T*>(At->vals)};
+  p.n = n;
+  p.m = m;
+  p.nnz_a = At->nnz;
+  p.nx = nx;
+  p.x_idx = x_idx;
+  p.x_vals = static_cast<const T*>(x_vals);
+  p.sum = reinterpret_cast<DevSummary*>(b + o_sum);
+  p.acc = reinterpret_cast<T*>(b + o_acc);
+  p.bits = reinterpret_cast<uint32_t*>(b + o_bits);
+  p.off = reinterpret_cast<int64_t*>(b + o_off);
+  p.first = reinterpret_cast<int64_t*>(b + o_first);
+  p.cnt = reinterpret_cast<int64_t*>(b + o_cnt);
+  p.partials = reinterpret_cast<int64_t*>(b + o_part);
+  p.y_idx = y_idx;
+  p.y_vals = static_cast<T*>(y_vals);
+  p.cap = m;
+  pl->dsum = p.sum;
+  pl->sym_launches = 0;
+  pl->num_launches = 0;
+  // zero the summary, the accumulator and the bitmap (contiguous), and the scan heads
+  WS_CUDA(cudaMemsetAsync(b, 0, o_off, s), "cudaMemsetAsync(spmspv scratch)");
+  WS_CUDA(cudaMemsetAsync(p.off, 0, sizeof(int64_t), s), "cudaMemsetAsync(off[0])");
+  WS_CUDA(cudaMemsetAsync(p.cnt, 0, sizeof(int64_t), s), "cudaMemsetAsync(cnt[0])");
+  if (m > 0) {
+    launch_spmspv<T>(p, num_sms_of(At->device), s, &pl->num_launches);
+    WS_CUDA(cudaGetLastError(), "spmspv launches");
+  }
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  st = device_status(*pl->host_sum);
+  if (st != WS_OK) return st;
+  *nnz_y = m > 0 ? pl->host_sum->nnz : 0;
+  return WS_OK;
+}
+
 // Shared checks of the operand and output handles; creates C's plan.
 ws_status_t prepare_output(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C) {
   if (C == A || C == B) return fail(WS_ERR_INVALID_ARG, "C must be a separate output handle");
@@ -704,6 +779,21 @@ ws_status_t ws_ewise_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_coli
   return WS_OK;
 }
 
+ws_status_t ws_spmspv(ws_csr_t At, int64_t nnz_x, const int32_t* x_idx, const void* x_vals, int32_t* y_idx,
+                      void* y_vals, int64_t* nnz_y, ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(At, "At")) != WS_OK) return st;
+  if (!nnz_y) return fail(WS_ERR_INVALID_ARG, "nnz_y is NULL");
+  if (nnz_x < 0 || nnz_x > At->nrows) return fail(WS_ERR_INVALID_ARG, "nnz_x must be in [0, %lld]", (long long)At->nrows);
+  if (nnz_x > 0 && (!x_idx || !x_vals)) return fail(WS_ERR_INVALID_ARG, "x_idx/x_vals NULL with nnz_x > 0");
+  if (At->ncols > 0 && (!y_idx || !y_vals)) return fail(WS_ERR_INVALID_ARG, "y_idx/y_vals NULL");
+  if ((st = ensure_plan(At)) != WS_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (At->dtype == WS_F64) return spmspv_impl<double>(At, nnz_x, x_idx, x_vals, y_idx, y_vals, nnz_y, s);
+  return spmspv_impl<float>(At, nnz_x, x_idx, x_vals, y_idx, y_vals, nnz_y, s);
+}
+
 ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
   g_last_error.clear();
   if (!C) return fail(WS_ERR_INVALID_ARG, "C is NULL");
@@ -721,11 +811,13 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
 ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
-    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr) cudaDeviceSynchronize();
+    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr || h->plan->sv.ptr)
+      cudaDeviceSynchronize();
     h->plan->rows.release();
     h->plan->slices.release();
     h->plan->ranks.release();
     h->plan->ew.release();
+    h->plan->sv.release();
     if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
     delete h->plan;
   }

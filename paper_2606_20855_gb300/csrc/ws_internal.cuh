@@ -175,6 +175,31 @@ void launch_ewise_symbolic(const EwisePlan<T>& p, int num_sms, cudaStream_t s, i
 template <typename T>
 void launch_ewise_numeric(const EwisePlan<T>& p, int num_sms, cudaStream_t s, int* launches);
 
+// Sparse matrix - sparse vector product y = A x, A given by columns (At = A^T in CSR).
+template <typename T>
+struct SpmspvPlan {
+  CsrView<T> At;         // n x m: row j holds column j of A
+  int64_t n;             // columns of A (rows of At)
+  int64_t m;             // rows of A = length of y
+  int64_t nnz_a;
+  int64_t nx;            // stored entries of x
+  const int32_t* x_idx;  // strictly increasing in [0, n)
+  const T* x_vals;
+  int64_t* off;          // [nx + 1]: products per x entry, then scanned in place
+  int64_t* first;        // [nx]: first entry of each x entry's column in At
+  T* acc;                // [m]: dense accumulator (zeroed by the host)
+  uint32_t* bits;        // [(m + 31) / 32]: positions of y hit (zeroed by the host)
+  int64_t* cnt;          // [tiles + 1]: set bits per compaction tile, then scanned in place
+  int64_t* partials;     // scan scratch for max(nx, tiles) entries
+  DevSummary* sum;
+  int32_t* y_idx;        // [cap]
+  T* y_vals;             // [cap]
+  int64_t cap;           // capacity of y (m)
+};
+int64_t spmspv_tiles(int64_t m);
+template <typename T>
+void launch_spmspv(const SpmspvPlan<T>& p, int num_sms, cudaStream_t s, int* launches);
+
 // Host-side launchers (one translation unit each).
 struct AnalyzeParams {
   int64_t m;

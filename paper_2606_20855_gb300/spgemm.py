@@ -190,6 +190,61 @@ def ewise(A: DeviceCSR, B: DeviceCSR, op: str = "add", validate: bool = False, s
     return C
 
 
+class SpMSpV:
+    """A reusable sparse matrix - sparse vector product y = A x, with A given by
+    columns: ``At`` is the DeviceCSR of A^T (row j of ``At`` = column j of A).
+
+    ``__call__(x_idx, x_vals)`` returns (y_idx, y_vals) as CUDA tensors (views
+    of capacity-m buffers kept by the object); it synchronises the stream.
+    """
+
+    def __init__(self, At: DeviceCSR, validate: bool = False, stream=None):
+        self.At = At
+        self._h = None
+        self._h = At._handle(validate, _stream_handle(stream))
+        dev = At.rowptr.device
+        self._y_idx = torch.empty(At.ncols, dtype=torch.int32, device=dev)
+        self._y_vals = torch.empty(At.ncols, dtype=At.dtype, device=dev)
+
+    def __call__(self, x_idx: torch.Tensor, x_vals: torch.Tensor, stream=None):
+        if x_idx.dtype != torch.int32 or x_vals.dtype != self.At.dtype or not x_idx.is_cuda or not x_vals.is_cuda:
+            raise TypeError("x_idx must be a CUDA int32 tensor and x_vals a CUDA tensor of A's dtype")
+        if x_idx.numel() != x_vals.numel():
+            raise ValueError("x_idx and x_vals differ in length")
+        x_idx, x_vals = x_idx.contiguous(), x_vals.contiguous()
+        nx = x_idx.numel()
+        nnz = _abi.ws_spmspv(self._h, nx, x_idx.data_ptr() if nx else 0, x_vals.data_ptr() if nx else 0,
+                             self._y_idx.data_ptr(), self._y_vals.data_ptr(), _stream_handle(stream))
+        return self._y_idx[:nnz], self._y_vals[:nnz]
+
+    def plan_info(self) -> dict:
+        return _abi.ws_spgemm_plan_info(self._h)
+
+    def close(self) -> None:
+        if self._h:
+            _abi.ws_csr_destroy(self._h)
+            self._h = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def spmspv(At: DeviceCSR, x_idx: torch.Tensor, x_vals: torch.Tensor, stream=None):
+    """y = A x for a sparse x (A given by columns: At = A^T in CSR); returns (y_idx, y_vals)."""
+    with SpMSpV(At, stream=stream) as op:
+        yi, yv = op(x_idx, x_vals, stream)
+        return yi.clone(), yv.clone()
+
+
 def spgemm(A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None) -> DeviceCSR:
     """C = A*B for CSR matrices on the GPU (sorted columns, structural zeros kept)."""
     with SpGEMM(A, B, validate=validate, stream=stream) as op:
