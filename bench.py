@@ -14,7 +14,9 @@ Extra keys: `e2e` (the same product through the public Python API from
 pinned host inputs to the host copy of C, copies inside the timed region),
 With an elementwise workload (``--workload ewise_* --op add|mul``) a step is
 one elementwise operation C = A + B or C = A .* B and the value is its
-effective bandwidth in GB/s of compulsory bytes.
+effective bandwidth in GB/s of compulsory bytes; with ``--workload spmspv_*``
+a step is one sparse matrix - sparse vector product y = A x (A resident by
+columns, x the step's input), also in GB/s of compulsory bytes.
 
 `roofline` (the whole product -- symbolic + numeric, the span the throughput
 target is set on -- against the measured copy bandwidth, with each pass's own
@@ -42,10 +44,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-from synth import EWISE_WORKLOADS, WORKLOADS, ewise_workload, workload  # noqa: E402
+from synth import EWISE_WORKLOADS, SPMSPV_WORKLOADS, WORKLOADS, ewise_workload, spmspv_workload, workload  # noqa: E402
 
 METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per config"
 EWISE_METRIC = "SpAdd / Hadamard effective HBM GB/s (compulsory bytes: read A and B, write C)"
+SPMSPV_METRIC = "SpMSpV effective HBM GB/s (compulsory bytes: read x, the columns of A it selects, write y)"
 DEFAULT_WORKLOAD = "uniform_rect_1m"
 NOMINAL_HBM_GBS = 8000.0
 
@@ -318,6 +321,128 @@ def run_reference_ewise(args) -> None:
     print(json.dumps(line), flush=True)
 
 
+def spmspv_bytes(At, x_idx, nnz_y: int) -> int:
+    """Compulsory bytes of y = A x: x, the column pointers and entries of the
+    columns x selects, and y."""
+    s = At.vals.dtype.itemsize
+    cols = np.asarray(x_idx, dtype=np.int64)
+    products = int((At.rowptr[cols + 1] - At.rowptr[cols]).sum())
+    return (4 + s) * cols.size + 16 * cols.size + (4 + s) * products + (4 + s) * nnz_y
+
+
+def run_spmspv(args, world, rank, local, pg) -> None:
+    import torch
+    from oracle import oracle_spmspv
+    from paper_2606_20855_gb300 import _abi
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpMSpV
+    from synth import transpose_csr
+
+    A, xi, xv = spmspv_workload(args.workload)
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        for _ in range(max(args.warmup, 0)):
+            oracle_spmspv(A, xi, xv)
+        times = []
+        for _ in range(max(args.steps, 1)):
+            t0 = time.perf_counter()
+            y = oracle_spmspv(A, xi, xv)
+            times.append(time.perf_counter() - t0)
+        At = transpose_csr(A)
+        dt = statistics.mean(times)
+        value = spmspv_bytes(At, xi, y.nnz) / dt / 1e9
+        line = {"impl": "reference", "metric": SPMSPV_METRIC, "value": round(value, 4), "unit": "GB/s",
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * dt, 3),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": args.workload, "description": SPMSPV_WORKLOADS[args.workload]},
+                "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                 "sample": "whole product, numpy on one core"},
+                "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return
+    _abi.load()
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    At = transpose_csr(A)
+    dAt = DeviceCSR.from_host(At, device)
+    dxi = torch.from_numpy(xi).to(device)
+    dxv = torch.from_numpy(xv).to(device)
+    stream = torch.cuda.current_stream(device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
+    op = SpMSpV(dAt)
+    for _ in range(args.warmup):
+        yi, _ = op(dxi, dxv)
+    nnz_y = int(yi.numel())
+    algo = spmspv_bytes(At, xi, nnz_y)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local).start() if rank == 0 else None
+    barrier(world, pg)
+    torch.cuda.synchronize(device)
+    t_wall0 = time.time()
+    for i in range(args.steps):
+        flush.fill_(i)  # write > L2 between timed steps (not timed)
+        ev[i][0].record(stream)
+        op(dxi, dxv)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(device)
+    t_wall1 = time.time()
+    barrier(world, pg)
+    clk = clocks.stop(t_wall0, t_wall1) if clocks else None
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_s = reduce_max(sum(step_ms) / 1e3, world, pg, device)
+    launches = op.plan_info()["numeric_launches"]
+    e2e = None
+    if args.e2e_steps > 0:
+        hxi, hxv = torch.from_numpy(xi).pin_memory(), torch.from_numpy(xv).pin_memory()
+        hyi = torch.empty(nnz_y, dtype=torch.int32).pin_memory()
+        hyv = torch.empty(nnz_y, dtype=torch.float64).pin_memory()
+
+        def e2e_step():
+            yi2, yv2 = op(hxi.to(device, non_blocking=True), hxv.to(device, non_blocking=True))
+            hyi.copy_(yi2, non_blocking=True)
+            hyv.copy_(yv2, non_blocking=True)
+            torch.cuda.synchronize(device)
+
+        e2e_step()
+        barrier(world, pg)
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2e_s = reduce_max(time.perf_counter() - t0, world, pg, device)
+        e2e = {"value": round(algo * args.e2e_steps * world / e2e_s / 1e9, 3), "unit": "GB/s",
+               "h2d_bytes_per_step": int(hxi.numel() * 4 + hxv.numel() * 8),
+               "d2h_bytes_per_step": int(nnz_y * 12), "steps": args.e2e_steps,
+               "note": "A stays resident (the operator); x is the step's input"}
+    op.close()
+    if rank != 0:
+        return
+    peaks = measured_peaks()
+    value = algo * args.steps * world / total_s / 1e9
+    base = None
+    if args.cpu_baseline_s > 0:
+        t0 = time.perf_counter()
+        oracle_spmspv(A, xi, xv)
+        dt = time.perf_counter() - t0
+        base = {"value": round(algo / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                "sample": f"whole product, {dt:.1f} s, numpy on one core"}
+    line = {
+        "metric": SPMSPV_METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(1e3 * total_s / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "description": SPMSPV_WORKLOADS[args.workload], "m": A.nrows,
+                   "n": A.ncols, "nnz_a": int(A.colidx.size), "nnz_x": int(xi.size), "nnz_y": nnz_y,
+                   "l2": "flushed between timed steps (write of a buffer > L2)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "phases_ms": {"step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
+        "roofline": dict(roofline_obj(algo, statistics.mean(step_ms) / 1e3, peaks, None),
+                         kernel="whole product (offsets, scan, scatter, tile counts, scan, write; read-back included)"),
+        "gpu_launches": int(launches * args.steps),
+        "clocks": clk, "e2e": e2e, "cpu_baseline": base,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_ours(args, world, rank, local, pg) -> None:
     import torch
     from paper_2606_20855_gb300 import _abi
@@ -495,7 +620,8 @@ def main(argv=None) -> int:
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=list(WORKLOADS) + list(EWISE_WORKLOADS), default=DEFAULT_WORKLOAD)
+    ap.add_argument("--workload", choices=list(WORKLOADS) + list(EWISE_WORKLOADS) + list(SPMSPV_WORKLOADS),
+                    default=DEFAULT_WORKLOAD)
     ap.add_argument("--op", choices=["add", "mul"], default="add", help="elementwise workloads: C = A + B or A .* B")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
@@ -507,7 +633,9 @@ def main(argv=None) -> int:
     args = ap.parse_args(argv)
     world, rank, local, pg = dist_setup()
     try:
-        if args.impl == "reference":
+        if args.workload in SPMSPV_WORKLOADS:
+            run_spmspv(args, world, rank, local, pg)
+        elif args.impl == "reference":
             run_reference(args, world, rank)
         else:
             run_ours(args, world, rank, local, pg)

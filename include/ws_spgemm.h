@@ -180,7 +180,7 @@ ws_status_t ws_ewise_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_coli
  * exactly 0.0 is kept), y[i] = sum of A[i,j] x[j] accumulated in the value
  * type in unspecified order.  Work is queued on `stream` and the call
  * synchronises it (to return nnz_y).  Device scratch (an accumulator and a
- * bitmap of length m, offsets per x entry) is allocated stream-ordered and
+ * byte-map of length m, offsets per x entry) is allocated stream-ordered and
  * cached in At's handle.  Errors: WS_ERR_INVALID_ARG (NULL pointers, nnz_x out
  * of range), WS_ERR_DEVICE (an index of x or of At out of range: those entries
  * are skipped and flagged).

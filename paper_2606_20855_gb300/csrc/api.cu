@@ -95,7 +95,7 @@ struct Plan {
   DevBuf slices;  // dense-window slice arrays
   DevBuf ranks;   // register bitmap rows: kBmrSlots uint16 ranks per row of A
   DevBuf ew;      // elementwise operations: summary, chunk arrays, scan partials
-  DevBuf sv;      // sparse matrix - sparse vector product (in A^T's handle): accumulator, bitmap, offsets
+  DevBuf sv;      // sparse matrix - sparse vector product (in A^T's handle): accumulator, byte-map, offsets
   int kind = kPlanNone;  // which symbolic pass filled this plan
   // elementwise plan (kPlanEwise)
   int ew_op = 0, ew_group = 32;
@@ -557,12 +557,12 @@ ws_status_t spmspv_impl(ws_csr_s* At, int64_t nx, const int32_t* x_idx, const vo
   Plan* pl = At->plan;
   const int64_t m = At->ncols, n = At->nrows;
   const int64_t tiles = spmspv_tiles(m);
-  const int64_t words = (m + 31) / 32;
+  const int64_t mark_bytes = tiles * 4096;  // the byte-map, padded to whole compaction tiles
   const int64_t nb = scan_partials_needed(nx > tiles ? nx : tiles);
   size_t off = 0;
   const size_t o_sum = off; off = align_up(off + sizeof(DevSummary), 256);
   const size_t o_acc = off; off = align_up(off + sizeof(T) * static_cast<size_t>(m), 256);
-  const size_t o_bits = off; off = align_up(off + 4 * static_cast<size_t>(words), 256);
+  const size_t o_mark = off; off = align_up(off + static_cast<size_t>(mark_bytes), 256);
   const size_t o_off = off; off = align_up(off + 8 * static_cast<size_t>(nx + 1), 256);
   const size_t o_first = off; off = align_up(off + 8 * static_cast<size_t>(nx), 256);
   const size_t o_cnt = off; off = align_up(off + 8 * static_cast<size_t>(tiles + 1), 256);
@@ -580,7 +580,7 @@ ws_status_t spmspv_impl(ws_csr_s* At, int64_t nx, const int32_t* x_idx, const vo
   p.x_vals = static_cast<const T*>(x_vals);
   p.sum = reinterpret_cast<DevSummary*>(b + o_sum);
   p.acc = reinterpret_cast<T*>(b + o_acc);
-  p.bits = reinterpret_cast<uint32_t*>(b + o_bits);
+  p.mark = reinterpret_cast<uint8_t*>(b + o_mark);
   p.off = reinterpret_cast<int64_t*>(b + o_off);
   p.first = reinterpret_cast<int64_t*>(b + o_first);
   p.cnt = reinterpret_cast<int64_t*>(b + o_cnt);
@@ -591,7 +591,7 @@ ws_status_t spmspv_impl(ws_csr_s* At, int64_t nx, const int32_t* x_idx, const vo
   pl->dsum = p.sum;
   pl->sym_launches = 0;
   pl->num_launches = 0;
-  // zero the summary, the accumulator and the bitmap (contiguous), and the scan heads
+  // zero the summary, the accumulator and the byte-map (contiguous), and the scan heads
   WS_CUDA(cudaMemsetAsync(b, 0, o_off, s), "cudaMemsetAsync(spmspv scratch)");
   WS_CUDA(cudaMemsetAsync(p.off, 0, sizeof(int64_t), s), "cudaMemsetAsync(off[0])");
   WS_CUDA(cudaMemsetAsync(p.cnt, 0, sizeof(int64_t), s), "cudaMemsetAsync(cnt[0])");

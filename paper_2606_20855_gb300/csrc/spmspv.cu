@@ -4,16 +4,16 @@
 // wrapped in a merge level because different columns hit the same positions
 // of y.  Here A is given by columns (the CSR of A^T), and the merge level is
 // the L2: every product is added into one dense accumulator of length m with
-// a global atomic add, and its position is marked in a bitmap (the byte-map
-// with a bit per position).  The coalesce step is a compaction of the bitmap
-// in index order.
+// a global atomic add, and its position is marked in a byte-map (a plain
+// store of 1: idempotent, so positions that many columns hit need no atomic).
+// The coalesce step is a compaction of the byte-map in index order.
 //
 //   1. product offsets: off[k + 1] = length of column x_idx[k] of A, and the
 //      column's first entry; scan -> off[k] = first product of x entry k
-//   2. scatter: product p (balanced over the GPU: every thread takes products
-//      p, p + stride, ...) finds its x entry by binary search in off, then
-//      acc[i] += A[i,j] x[j] and sets bit i
-//   3. compaction: set bits per tile of 4096 positions -> scan -> every tile
+//   2. scatter: tiles of consecutive products (balanced over the GPU) find
+//      the x entries they span, and every product finds its entry by binary
+//      search in those offsets, then acc[i] += A[i,j] x[j] and mark[i] = 1
+//   3. compaction: marks per tile of 4096 positions -> scan -> every tile
 //      writes its positions (ascending) and accumulated values to y
 #include "ws_internal.cuh"
 
@@ -22,7 +22,13 @@ namespace wsk {
 namespace {
 
 constexpr int kSvThreads = 256;
-constexpr int kSvTile = 4096;  // positions of y per compaction tile (128 bitmap words)
+constexpr int kSvTile = 4096;  // positions of y per compaction tile (4 KB of the byte-map)
+
+// Counts the non-zero bytes of 16 bytes.
+__device__ __forceinline__ int marked(const uint4 v) {
+  return __popc(__vcmpne4(v.x, 0u) & 0x01010101u) + __popc(__vcmpne4(v.y, 0u) & 0x01010101u) +
+         __popc(__vcmpne4(v.z, 0u) & 0x01010101u) + __popc(__vcmpne4(v.w, 0u) & 0x01010101u);
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kSvThreads) sv_offsets_kernel(const SpmspvPlan<T> p) {
@@ -41,41 +47,127 @@ __global__ void __launch_bounds__(kSvThreads) sv_offsets_kernel(const SpmspvPlan
   }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kSvThreads) sv_scatter_kernel(const SpmspvPlan<T> p) {
-  const int64_t total = p.off[p.nx];
-  for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < total;
-       q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    // x entry k with off[k] <= q < off[k + 1] (off is non-decreasing; the last k wins for empty columns)
-    int64_t lo = 0, hi = p.nx - 1;
-    while (lo < hi) {  // O(log nx) probes
-      const int64_t mid = (lo + hi + 1) >> 1;
-      if (p.off[mid] <= q) {
-        lo = mid;
-      } else {
-        hi = mid - 1;
-      }
-    }
-    const int64_t b = p.first[lo] + (q - p.off[lo]);
-    const int32_t i = p.At.colidx[b];
-    if (i < 0 || i >= p.m) {
-      atomicOr(&p.sum->status, kErrCount);
-      continue;
-    }
-    atomicAdd(p.acc + i, p.At.vals[b] * p.x_vals[lo]);
-    atomicOr(p.bits + (i >> 5), 1u << (i & 31));
+// Largest k in [lo, hi] with off[k] <= q, given off[lo] <= q; a 32-way search
+// by one warp (every lane probes one point per level).  O(log_32 (hi - lo)) levels.
+__device__ __forceinline__ int64_t warp_last_le(const int64_t* off, int64_t lo, int64_t hi, int64_t q) {
+  const int lane = threadIdx.x & 31;
+  for (int level = 0; level < 16 && hi > lo; ++level) {
+    const int64_t step = (hi - lo + 32) / 32;
+    const int64_t pos = lo + lane * step;
+    const unsigned m = __ballot_sync(0xffffffffu, pos <= hi && off[pos] <= q);
+    lo += static_cast<int64_t>(31 - __clz(m)) * step;  // lane 0 always qualifies
+    hi = hi < lo + step - 1 ? hi : lo + step - 1;
   }
+  return lo;
 }
 
-// Set bits of every compaction tile: cnt[t + 1].
-__global__ void __launch_bounds__(kSvThreads) sv_tile_count_kernel(const uint32_t* bits, int64_t m, int64_t* cnt) {
+// Load-balanced scatter: a CTA takes kScatterTile consecutive products, two
+// warps find the x entries holding the first and the last, the offsets of
+// that range go to shared memory (when it fits), and every thread finds the
+// entry of each of its products by binary search there.
+constexpr int kPerThread = 8;
+constexpr int kScatterTile = kSvThreads * kPerThread;
+constexpr int kScatterSpan = 2048;  // x entries of one tile kept in shared memory
+
+template <typename T>
+__global__ void __launch_bounds__(kSvThreads) sv_scatter_kernel(const SpmspvPlan<T> p) {
+  __shared__ long long s_off[kScatterSpan + 1];
+  __shared__ long long s_k[2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t total = p.off[p.nx];
+  bool bad = false;
+  for (int64_t t0 = static_cast<int64_t>(blockIdx.x) * kScatterTile; t0 < total;
+       t0 += static_cast<int64_t>(gridDim.x) * kScatterTile) {
+    const int64_t t1 = t0 + kScatterTile < total ? t0 + kScatterTile : total;
+    if (warp < 2) {
+      const int64_t k = warp_last_le(p.off, 0, p.nx - 1, warp == 0 ? t0 : t1 - 1);
+      if (lane == 0) s_k[warp] = k;
+    }
+    __syncthreads();
+    const int64_t k0 = s_k[0], k1 = s_k[1];
+    const bool in_smem = k1 - k0 + 1 <= kScatterSpan;
+    if (in_smem) {
+      for (int64_t i = threadIdx.x; i <= k1 - k0 + 1; i += blockDim.x) s_off[i] = p.off[k0 + i];
+    }
+    __syncthreads();
+    // Each thread takes kPerThread products of the tile; the lookups come
+    // first, then every load is issued before the first add, so the loads of
+    // all its products are in flight together.
+    int64_t kk[kPerThread], bb[kPerThread];
+#pragma unroll
+    for (int r = 0; r < kPerThread; ++r) {
+      const int64_t q = t0 + threadIdx.x + static_cast<int64_t>(r) * kSvThreads;
+      kk[r] = -1;
+      bb[r] = 0;
+      if (q < t1) {
+        int64_t k;
+        if (in_smem) {  // largest local index with s_off <= q
+          int lo = 0, hi = static_cast<int>(k1 - k0);
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_off[mid] <= q) {
+              lo = mid;
+            } else {
+              hi = mid - 1;
+            }
+          }
+          k = k0 + lo;
+          bb[r] = q - s_off[lo];
+        } else {
+          int64_t lo = k0, hi = k1;
+          while (lo < hi) {
+            const int64_t mid = (lo + hi + 1) >> 1;
+            if (p.off[mid] <= q) {
+              lo = mid;
+            } else {
+              hi = mid - 1;
+            }
+          }
+          k = lo;
+          bb[r] = q - p.off[lo];
+        }
+        kk[r] = k;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < kPerThread; ++r) {
+      if (kk[r] >= 0) bb[r] += p.first[kk[r]];
+    }
+    int32_t ii[kPerThread];
+    T vv[kPerThread];
+#pragma unroll
+    for (int r = 0; r < kPerThread; ++r) {
+      ii[r] = -1;
+      vv[r] = T(0);
+      if (kk[r] >= 0) {
+        ii[r] = p.At.colidx[bb[r]];
+        vv[r] = p.At.vals[bb[r]] * p.x_vals[kk[r]];
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < kPerThread; ++r) {
+      if (kk[r] < 0) continue;
+      const int32_t i = ii[r];
+      if (i < 0 || i >= p.m) {
+        bad = true;
+        continue;
+      }
+      atomicAdd(p.acc + i, vv[r]);
+      p.mark[i] = 1;
+    }
+    __syncthreads();  // s_off and s_k are reused by the next tile
+  }
+  if (bad) atomicOr(&p.sum->status, kErrCount);
+}
+
+// Marked positions of every compaction tile: cnt[t + 1].  One thread reads 16
+// bytes (the byte-map is padded to whole tiles with zeros).
+__global__ void __launch_bounds__(kSvThreads) sv_tile_count_kernel(const uint8_t* mark, int64_t m, int64_t* cnt) {
+  static_assert(kSvTile == kSvThreads * 16, "one 16-byte load per thread and tile");
   __shared__ int s_red[kSvThreads / 32];
-  const int64_t words = (m + 31) >> 5;
   const int64_t tiles = (m + kSvTile - 1) / kSvTile;
   for (int64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
-    const int64_t w0 = t * (kSvTile / 32);
-    int c = 0;
-    for (int64_t w = w0 + threadIdx.x; w < w0 + kSvTile / 32 && w < words; w += blockDim.x) c += __popc(bits[w]);
+    int c = marked(reinterpret_cast<const uint4*>(mark + t * kSvTile)[threadIdx.x]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
     if ((threadIdx.x & 31) == 0) s_red[threadIdx.x >> 5] = c;
@@ -89,20 +181,18 @@ __global__ void __launch_bounds__(kSvThreads) sv_tile_count_kernel(const uint32_
   }
 }
 
-// Tile t writes its set positions in ascending order from y offset cnt[t]:
-// one warp per 32-word slice of the tile, ballots give the order.
+// Tile t writes its marked positions in ascending order from y offset
+// cnt[t]: warp w takes the tile's positions [512 w, 512 w + 512) in 16 rounds
+// of 32, and ballots give the order.
 template <typename T>
 __global__ void __launch_bounds__(kSvThreads) sv_write_kernel(const SpmspvPlan<T> p) {
+  constexpr int kPerWarp = kSvTile / (kSvThreads / 32);  // 512
   __shared__ long long s_base[kSvThreads / 32 + 1];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t words = (p.m + 31) >> 5;
   const int64_t tiles = (p.m + kSvTile - 1) / kSvTile;
   for (int64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
-    // the tile's 128 words: warp w takes words [w0 + 16w, w0 + 16w + 16)
-    constexpr int kWordsPerWarp = kSvTile / 32 / (kSvThreads / 32);
-    const int64_t w0 = t * (kSvTile / 32) + static_cast<int64_t>(warp) * kWordsPerWarp;
-    int c = 0;
-    if (lane < kWordsPerWarp && w0 + lane < words) c = __popc(p.bits[w0 + lane]);
+    const int64_t i0 = t * kSvTile + static_cast<int64_t>(warp) * kPerWarp;
+    int c = marked(reinterpret_cast<const uint4*>(p.mark + i0)[lane]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
     if (lane == 0) s_base[warp + 1] = c;
@@ -114,21 +204,20 @@ __global__ void __launch_bounds__(kSvThreads) sv_write_kernel(const SpmspvPlan<T
     __syncthreads();
     long long pos = s_base[warp];
     const long long end = p.cnt[t + 1];
-    for (int q = 0; q < kWordsPerWarp; ++q) {
-      const int64_t w = w0 + q;
-      const uint32_t word = w < words ? p.bits[w] : 0u;  // same word for every lane
-      const bool set = (word >> lane) & 1u;
+    for (int q = 0; q < kPerWarp / 32; ++q) {
+      const int64_t i = i0 + q * 32 + lane;
+      const bool set = p.mark[i] != 0;
+      const unsigned bal = __ballot_sync(0xffffffffu, set);
       if (set) {
-        const long long at = pos + __popc(word & ((1u << lane) - 1u));
-        const int64_t i = (w << 5) + lane;
-        if (at < end && at < p.cap) {
+        const long long at = pos + __popc(bal & ((1u << lane) - 1u));
+        if (at < end && at < p.cap && i < p.m) {
           p.y_idx[at] = static_cast<int32_t>(i);
           p.y_vals[at] = p.acc[i];
         } else {
           atomicOr(&p.sum->status, kErrCount);
         }
       }
-      pos += __popc(word);
+      pos += __popc(bal);
     }
     __syncthreads();
   }
@@ -150,11 +239,11 @@ void launch_spmspv(const SpmspvPlan<T>& p, int num_sms, cudaStream_t s, int* lau
     sv_offsets_kernel<T><<<grid_for(p.nx, kSvThreads, num_sms, 8), kSvThreads, 0, s>>>(p);
     launch_scan(p.off, p.nx, p.partials, p.sum, s, launches);
     // products are at most nnz(A); the kernel stops at the scanned total
-    sv_scatter_kernel<T><<<grid_for(p.nnz_a, kSvThreads, num_sms, 8), kSvThreads, 0, s>>>(p);
+    sv_scatter_kernel<T><<<grid_for(p.nnz_a, kScatterTile, num_sms, 8), kSvThreads, 0, s>>>(p);
     *launches += 2;
   }
   const int64_t tiles = spmspv_tiles(p.m);
-  sv_tile_count_kernel<<<grid_for(tiles, 1, num_sms, 8), kSvThreads, 0, s>>>(p.bits, p.m, p.cnt);
+  sv_tile_count_kernel<<<grid_for(tiles, 1, num_sms, 8), kSvThreads, 0, s>>>(p.mark, p.m, p.cnt);
   launch_scan(p.cnt, tiles, p.partials, p.sum, s, launches);
   sv_write_kernel<T><<<grid_for(tiles, 1, num_sms, 8), kSvThreads, 0, s>>>(p);
   *launches += 2;

@@ -188,7 +188,7 @@ struct SpmspvPlan {
   int64_t* off;          // [nx + 1]: products per x entry, then scanned in place
   int64_t* first;        // [nx]: first entry of each x entry's column in At
   T* acc;                // [m]: dense accumulator (zeroed by the host)
-  uint32_t* bits;        // [(m + 31) / 32]: positions of y hit (zeroed by the host)
+  uint8_t* mark;         // [tiles * 4096]: 1 at the positions of y hit (zeroed by the host)
   int64_t* cnt;          // [tiles + 1]: set bits per compaction tile, then scanned in place
   int64_t* partials;     // scan scratch for max(nx, tiles) entries
   DevSummary* sum;
