@@ -189,6 +189,23 @@ ws_status_t ws_spmspv(ws_csr_t At, int64_t nnz_x, const int32_t* x_idx, const vo
                       void* y_vals, int64_t* nnz_y, ws_stream_t stream);
 
 /*
+ * ws_csr_submatrix_symbolic / ws_csr_submatrix_numeric -- S = A[r0:r1, c0:c1]
+ * as a CSR matrix of shape (r1 - r0) x (c1 - c0) with columns shifted by -c0.
+ * This is the layout step of the outer-product SpGEMM (Sec. 5.1, Fig.
+ * "SpGEMM implemented in WingSpan": the k loop split over workers, worker p
+ * multiplying the column block A[:, K_p] by the row block B[K_p, :] into its
+ * own copy of C before a merge level coalesces the copies).
+ *   0 <= r0 <= r1 <= A.nrows, 0 <= c0 <= c1 <= A.ncols (else WS_ERR_INVALID_ARG)
+ *   S   output handle of shape (r1 - r0) x (c1 - c0) and A's dtype
+ * The symbolic call writes S.rowptr and returns nnz(S) (it synchronises
+ * `stream`); the numeric call (asynchronous) fills the caller's s_colidx
+ * (int32[nnz(S)]) and s_vals from the same A, unchanged in between.
+ */
+ws_status_t ws_csr_submatrix_symbolic(ws_csr_t A, int64_t r0, int64_t r1, int64_t c0, int64_t c1, ws_csr_t S,
+                                      int64_t* nnz_out, ws_stream_t stream);
+ws_status_t ws_csr_submatrix_numeric(ws_csr_t A, ws_csr_t S, int32_t* s_colidx, void* s_vals, ws_stream_t stream);
+
+/*
  * ws_spgemm_wait -- synchronises `stream` and returns the device status
  * recorded by the last symbolic/numeric pass of C (WS_OK if none failed);
  * serves the elementwise passes too.

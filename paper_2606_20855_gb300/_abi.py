@@ -46,6 +46,8 @@ SIGNATURES = [
     ("ws_ewise_symbolic", _i32, [_p, _p, _p, _i32, ctypes.POINTER(_i64), _p]),
     ("ws_ewise_numeric", _i32, [_p, _p, _p, _p, _p, _p]),
     ("ws_spmspv", _i32, [_p, _i64, _p, _p, _p, _p, ctypes.POINTER(_i64), _p]),
+    ("ws_csr_submatrix_symbolic", _i32, [_p, _i64, _i64, _i64, _i64, _p, ctypes.POINTER(_i64), _p]),
+    ("ws_csr_submatrix_numeric", _i32, [_p, _p, _p, _p, _p]),
 ]
 
 EWISE_OPS = {"add": 1, "mul": 2}  # ws_ewise_op_t
@@ -124,6 +126,18 @@ def ws_spmspv(At: int, nnz_x: int, x_idx: int, x_vals: int, y_idx: int, y_vals: 
     _check("ws_spmspv", load().ws_spmspv(At, nnz_x, x_idx or None, x_vals or None, y_idx or None, y_vals or None,
                                          ctypes.byref(nnz), stream or None))
     return nnz.value
+
+
+def ws_csr_submatrix_symbolic(A: int, r0: int, r1: int, c0: int, c1: int, S: int, stream: int) -> int:
+    nnz = ctypes.c_int64(-1)
+    _check("ws_csr_submatrix_symbolic", load().ws_csr_submatrix_symbolic(A, r0, r1, c0, c1, S, ctypes.byref(nnz),
+                                                                         stream or None))
+    return nnz.value
+
+
+def ws_csr_submatrix_numeric(A: int, S: int, s_colidx: int, s_vals: int, stream: int) -> None:
+    _check("ws_csr_submatrix_numeric", load().ws_csr_submatrix_numeric(A, S, s_colidx or None, s_vals or None,
+                                                                       stream or None))
 
 
 def ws_spgemm_wait(C: int, stream: int) -> None:

@@ -88,7 +88,7 @@ struct DevBuf {
   }
 };
 
-enum PlanKind { kPlanNone = 0, kPlanSpgemm = 1, kPlanEwise = 2 };
+enum PlanKind { kPlanNone = 0, kPlanSpgemm = 1, kPlanEwise = 2, kPlanSub = 3 };
 
 struct Plan {
   DevBuf rows;    // per-row arrays + summary + scan partials
@@ -104,6 +104,8 @@ struct Plan {
   int32_t* ew_chunk_row = nullptr;
   int64_t* ew_chunk_off = nullptr;
   int64_t* ew_partials = nullptr;
+  // submatrix plan (kPlanSub): the block the symbolic pass counted
+  int64_t sub_r0 = 0, sub_r1 = 0, sub_c0 = 0, sub_c1 = 0;
   DevSummary* host_sum = nullptr;  // pinned
   // carved pointers
   DevSummary* dsum = nullptr;
@@ -792,6 +794,88 @@ ws_status_t ws_spmspv(ws_csr_t At, int64_t nnz_x, const int32_t* x_idx, const vo
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (At->dtype == WS_F64) return spmspv_impl<double>(At, nnz_x, x_idx, x_vals, y_idx, y_vals, nnz_y, s);
   return spmspv_impl<float>(At, nnz_x, x_idx, x_vals, y_idx, y_vals, nnz_y, s);
+}
+
+ws_status_t ws_csr_submatrix_symbolic(ws_csr_t A, int64_t r0, int64_t r1, int64_t c0, int64_t c1, ws_csr_t S,
+                                      int64_t* nnz_out, ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(S, "S")) != WS_OK) return st;
+  if (!nnz_out) return fail(WS_ERR_INVALID_ARG, "nnz_out is NULL");
+  if (S == A) return fail(WS_ERR_INVALID_ARG, "S must be a separate output handle");
+  if (r0 < 0 || r0 > r1 || r1 > A->nrows || c0 < 0 || c0 > c1 || c1 > A->ncols)
+    return fail(WS_ERR_INVALID_ARG, "block [%lld:%lld, %lld:%lld] outside the %lldx%lld matrix", (long long)r0,
+                (long long)r1, (long long)c0, (long long)c1, (long long)A->nrows, (long long)A->ncols);
+  if (S->nrows != r1 - r0 || S->ncols != c1 - c0)
+    return fail(WS_ERR_SHAPE, "S is %lldx%lld, expected %lldx%lld", (long long)S->nrows, (long long)S->ncols,
+                (long long)(r1 - r0), (long long)(c1 - c0));
+  if (S->dtype != A->dtype) return fail(WS_ERR_DTYPE, "A and S dtypes differ");
+  if ((st = ensure_plan(S)) != WS_OK) return st;
+  Plan* pl = S->plan;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int64_t rows = r1 - r0;
+  const int64_t nb = scan_partials_needed(rows);
+  const size_t o_part = align_up(sizeof(DevSummary), 256);
+  if ((st = pl->ew.reserve(o_part + 8 * static_cast<size_t>(nb + 1), s)) != WS_OK) return st;
+  char* b = static_cast<char*>(pl->ew.ptr);
+  pl->dsum = reinterpret_cast<DevSummary*>(b);
+  int64_t* partials = reinterpret_cast<int64_t*>(b + o_part);
+  pl->ready = false;
+  pl->kind = kPlanSub;
+  pl->sym_launches = 0;
+  pl->num_launches = 0;
+  S->nnz = -1;
+  WS_CUDA(cudaMemsetAsync(pl->dsum, 0, sizeof(DevSummary), s), "cudaMemsetAsync(summary)");
+  WS_CUDA(cudaMemsetAsync(S->rowptr, 0, sizeof(int64_t), s), "cudaMemsetAsync(rowptr[0])");
+  if (rows > 0) {
+    const int sms = num_sms_of(S->device);
+    launch_submatrix_count(A->rowptr, A->colidx, r0, rows, c0, c1, S->rowptr, sms, s, &pl->sym_launches);
+    launch_scan(S->rowptr, rows, partials, pl->dsum, s, &pl->sym_launches);
+    WS_CUDA(cudaGetLastError(), "submatrix symbolic launches");
+  }
+  st = read_summary(pl, s);
+  if (st != WS_OK) return st;
+  S->nnz = rows > 0 ? pl->host_sum->nnz : 0;
+  pl->A = A;
+  pl->B = nullptr;
+  pl->a_nnz = A->nnz;
+  pl->sub_r0 = r0;
+  pl->sub_r1 = r1;
+  pl->sub_c0 = c0;
+  pl->sub_c1 = c1;
+  pl->ready = true;
+  *nnz_out = S->nnz;
+  return WS_OK;
+}
+
+ws_status_t ws_csr_submatrix_numeric(ws_csr_t A, ws_csr_t S, int32_t* s_colidx, void* s_vals, ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(S, "S")) != WS_OK) return st;
+  Plan* pl = S->plan;
+  if (!pl || !pl->ready || pl->kind != kPlanSub)
+    return fail(WS_ERR_STATE, "numeric called before a successful submatrix symbolic pass");
+  if (pl->A != A || pl->a_nnz != A->nnz)
+    return fail(WS_ERR_STATE, "numeric called with another matrix than the symbolic pass");
+  if (S->nnz > 0 && (!s_colidx || !s_vals)) return fail(WS_ERR_INVALID_ARG, "s_colidx/s_vals NULL with nnz(S) > 0");
+  S->colidx = s_colidx;
+  S->vals = s_vals;
+  pl->num_launches = 0;
+  if (S->nnz == 0) return WS_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int sms = num_sms_of(S->device);
+  const int64_t rows = pl->sub_r1 - pl->sub_r0;
+  if (A->dtype == WS_F64) {
+    launch_submatrix_copy<double>(A->rowptr, A->colidx, static_cast<const double*>(A->vals), pl->sub_r0, rows,
+                                  pl->sub_c0, S->rowptr, s_colidx, static_cast<double*>(s_vals), pl->dsum, sms, s,
+                                  &pl->num_launches);
+  } else {
+    launch_submatrix_copy<float>(A->rowptr, A->colidx, static_cast<const float*>(A->vals), pl->sub_r0, rows,
+                                 pl->sub_c0, S->rowptr, s_colidx, static_cast<float*>(s_vals), pl->dsum, sms, s,
+                                 &pl->num_launches);
+  }
+  WS_CUDA(cudaGetLastError(), "submatrix numeric launch");
+  return WS_OK;
 }
 
 ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {

@@ -200,6 +200,14 @@ int64_t spmspv_tiles(int64_t m);
 template <typename T>
 void launch_spmspv(const SpmspvPlan<T>& p, int num_sms, cudaStream_t s, int* launches);
 
+// Submatrix S = A[r0:r1, c0:c1]: per-row counts into s_rowptr[1..rows], then the copy.
+void launch_submatrix_count(const int64_t* rowptr, const int32_t* colidx, int64_t r0, int64_t rows, int64_t c0,
+                            int64_t c1, int64_t* s_rowptr, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_submatrix_copy(const int64_t* rowptr, const int32_t* colidx, const T* vals, int64_t r0, int64_t rows,
+                           int64_t c0, const int64_t* s_rowptr, int32_t* s_colidx, T* s_vals, DevSummary* sum,
+                           int num_sms, cudaStream_t s, int* launches);
+
 // Host-side launchers (one translation unit each).
 struct AnalyzeParams {
   int64_t m;

@@ -245,6 +245,51 @@ def spmspv(At: DeviceCSR, x_idx: torch.Tensor, x_vals: torch.Tensor, stream=None
         return yi.clone(), yv.clone()
 
 
+def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None) -> DeviceCSR:
+    """S = A[r0:r1, c0:c1] as a DeviceCSR with columns shifted by -c0 (CUDA kernels)."""
+    s = _stream_handle(stream)
+    hA = hS = None
+    try:
+        hA = A._handle(False, s)
+        rowptr = torch.empty(max(r1 - r0, 0) + 1, dtype=torch.int64, device=A.rowptr.device)
+        hS = _abi.ws_csr_create(r1 - r0, c1 - c0, 0, rowptr.data_ptr(), 0, 0, _DTYPES[A.dtype], False, s)
+        nnz = _abi.ws_csr_submatrix_symbolic(hA, r0, r1, c0, c1, hS, s)
+        colidx = torch.empty(nnz, dtype=torch.int32, device=A.rowptr.device)
+        vals = torch.empty(nnz, dtype=A.dtype, device=A.rowptr.device)
+        _abi.ws_csr_submatrix_numeric(hA, hS, colidx.data_ptr() if nnz else 0, vals.data_ptr() if nnz else 0, s)
+        _abi.ws_spgemm_wait(hS, s)
+        return DeviceCSR(r1 - r0, c1 - c0, rowptr, colidx, vals)
+    finally:
+        for h in (hS, hA):
+            if h:
+                _abi.ws_csr_destroy(h)
+
+
+def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None) -> DeviceCSR:
+    """C = A*B as the outer-product SpGEMM of Sec. 5.1: the k range is split
+    into `parts` contiguous blocks, block p contributes the partial product
+    A[:, K_p] * B[K_p, :] (a worker's own copy of C, computed by the row-wise
+    kernels), and the partial products are coalesced by pairwise sparse
+    additions (the merge level).  Same structure as spgemm(); values equal
+    up to summation order."""
+    if A.ncols != B.nrows:
+        raise ValueError(f"shape mismatch: A is {A.nrows}x{A.ncols}, B is {B.nrows}x{B.ncols}")
+    K = A.ncols
+    parts = max(1, min(int(parts), max(K, 1)))
+    bounds = [(K * p // parts, K * (p + 1) // parts) for p in range(parts)]
+    partial = []
+    for k0, k1 in bounds:
+        Ap = submatrix(A, 0, A.nrows, k0, k1, stream)
+        Bp = submatrix(B, k0, k1, 0, B.ncols, stream)
+        partial.append(spgemm(Ap, Bp, stream=stream))
+    while len(partial) > 1:
+        merged = [ewise(partial[i], partial[i + 1], "add", stream=stream) for i in range(0, len(partial) - 1, 2)]
+        if len(partial) % 2:
+            merged.append(partial[-1])
+        partial = merged
+    return partial[0]
+
+
 def spgemm(A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None) -> DeviceCSR:
     """C = A*B for CSR matrices on the GPU (sorted columns, structural zeros kept)."""
     with SpGEMM(A, B, validate=validate, stream=stream) as op:
