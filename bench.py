@@ -443,6 +443,58 @@ def run_spmspv(args, world, rank, local, pg) -> None:
     print(json.dumps(line), flush=True)
 
 
+def run_outer(args, world, rank, local, pg, A, B, dA, dB, ub, flush, stream, device) -> None:
+    """The outer-product SpGEMM (k blocks, partial products, sparse-addition merge), timed whole."""
+    import torch
+    from paper_2606_20855_gb300.spgemm import spgemm_outer
+    products = int(ub.sum())
+    C = None
+    for _ in range(args.warmup):
+        C = spgemm_outer(dA, dB, args.parts)
+    torch.cuda.synchronize(device)
+    nnz = C.nnz if C is not None else 0
+    stats = {}
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local).start() if rank == 0 else None
+    barrier(world, pg)
+    torch.cuda.synchronize(device)
+    t_wall0 = time.time()
+    for i in range(args.steps):
+        flush.fill_(i)
+        ev[i][0].record(stream)
+        C = spgemm_outer(dA, dB, args.parts, stats=stats)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(device)
+    t_wall1 = time.time()
+    barrier(world, pg)
+    clk = clocks.stop(t_wall0, t_wall1) if clocks else None
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_s = reduce_max(sum(step_ms) / 1e3, world, pg, device)
+    if rank != 0:
+        return
+    s = A.vals.dtype.itemsize
+    algo = csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz, s)
+    peaks = measured_peaks()
+    value = 2.0 * products * args.steps * world / total_s / 1e9
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "GFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(1e3 * total_s / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64" if s == 8 else "f32", "data": "synthetic",
+        "config": {"workload": args.workload, "description": WORKLOADS[args.workload], "algo": "outer",
+                   "parts": args.parts, "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_c": int(nnz),
+                   "products": products, "l2": "flushed between timed steps (write of a buffer > L2)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "effective_hbm_gbs": round(algo * args.steps * world / total_s / 1e9, 1),
+        "phases_ms": {"step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
+        "roofline": dict(roofline_obj(algo, statistics.mean(step_ms) / 1e3, peaks, None),
+                         kernel=f"whole outer-product SpGEMM ({args.parts} k blocks: submatrices, partial products, "
+                                "pairwise sparse additions; read-backs included)"),
+        "gpu_launches": int(stats.get("launches", 0)),
+        "clocks": clk, "e2e": None, "cpu_baseline": None,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_ours(args, world, rank, local, pg) -> None:
     import torch
     from paper_2606_20855_gb300 import _abi
@@ -465,6 +517,9 @@ def run_ours(args, world, rank, local, pg) -> None:
     l2 = torch.cuda.get_device_properties(device).L2_cache_size
     flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
 
+    if args.algo == "outer" and not ew:
+        run_outer(args, world, rank, local, pg, A, B, dA, dB, ub, flush, stream, device)
+        return
     op = make_op(dA, dB)
     out = None
 
@@ -623,6 +678,9 @@ def main(argv=None) -> int:
     ap.add_argument("--workload", choices=list(WORKLOADS) + list(EWISE_WORKLOADS) + list(SPMSPV_WORKLOADS),
                     default=DEFAULT_WORKLOAD)
     ap.add_argument("--op", choices=["add", "mul"], default="add", help="elementwise workloads: C = A + B or A .* B")
+    ap.add_argument("--algo", choices=["gustavson", "outer"], default="gustavson",
+                    help="SpGEMM workloads: row-wise (default) or the outer-product variant")
+    ap.add_argument("--parts", type=int, default=4, help="k blocks of the outer-product variant")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-baseline-s", type=float, default=12.0, help="seconds of CPU oracle work (0 = skip)")
     ap.add_argument("--ref-step-s", type=float, default=2.0, help="seconds per reference-arm step")

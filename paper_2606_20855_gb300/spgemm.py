@@ -245,8 +245,9 @@ def spmspv(At: DeviceCSR, x_idx: torch.Tensor, x_vals: torch.Tensor, stream=None
         return yi.clone(), yv.clone()
 
 
-def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None) -> DeviceCSR:
-    """S = A[r0:r1, c0:c1] as a DeviceCSR with columns shifted by -c0 (CUDA kernels)."""
+def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None, stats: dict | None = None) -> DeviceCSR:
+    """S = A[r0:r1, c0:c1] as a DeviceCSR with columns shifted by -c0 (CUDA kernels).
+    `stats["launches"]`, when given, is increased by the kernel launches queued."""
     s = _stream_handle(stream)
     hA = hS = None
     try:
@@ -258,6 +259,9 @@ def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None) -> 
         vals = torch.empty(nnz, dtype=A.dtype, device=A.rowptr.device)
         _abi.ws_csr_submatrix_numeric(hA, hS, colidx.data_ptr() if nnz else 0, vals.data_ptr() if nnz else 0, s)
         _abi.ws_spgemm_wait(hS, s)
+        if stats is not None:
+            info = _abi.ws_spgemm_plan_info(hS)
+            stats["launches"] = stats.get("launches", 0) + info["symbolic_launches"] + info["numeric_launches"]
         return DeviceCSR(r1 - r0, c1 - c0, rowptr, colidx, vals)
     finally:
         for h in (hS, hA):
@@ -265,13 +269,24 @@ def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None) -> 
                 _abi.ws_csr_destroy(h)
 
 
-def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None) -> DeviceCSR:
+def _run(op, stats: dict | None, stream=None) -> DeviceCSR:
+    with op:
+        op.symbolic(stream)
+        C = op.numeric(stream=stream)
+        op.wait(stream)
+        if stats is not None:
+            info = op.plan_info()
+            stats["launches"] = stats.get("launches", 0) + info["symbolic_launches"] + info["numeric_launches"]
+    return C
+
+
+def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None, stats: dict | None = None) -> DeviceCSR:
     """C = A*B as the outer-product SpGEMM of Sec. 5.1: the k range is split
     into `parts` contiguous blocks, block p contributes the partial product
     A[:, K_p] * B[K_p, :] (a worker's own copy of C, computed by the row-wise
     kernels), and the partial products are coalesced by pairwise sparse
     additions (the merge level).  Same structure as spgemm(); values equal
-    up to summation order."""
+    up to summation order.  `stats["launches"]` counts the kernel launches."""
     if A.ncols != B.nrows:
         raise ValueError(f"shape mismatch: A is {A.nrows}x{A.ncols}, B is {B.nrows}x{B.ncols}")
     K = A.ncols
@@ -279,11 +294,12 @@ def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None) -> Dev
     bounds = [(K * p // parts, K * (p + 1) // parts) for p in range(parts)]
     partial = []
     for k0, k1 in bounds:
-        Ap = submatrix(A, 0, A.nrows, k0, k1, stream)
-        Bp = submatrix(B, k0, k1, 0, B.ncols, stream)
-        partial.append(spgemm(Ap, Bp, stream=stream))
+        Ap = submatrix(A, 0, A.nrows, k0, k1, stream, stats)
+        Bp = submatrix(B, k0, k1, 0, B.ncols, stream, stats)
+        partial.append(_run(SpGEMM(Ap, Bp, stream=stream), stats, stream))
     while len(partial) > 1:
-        merged = [ewise(partial[i], partial[i + 1], "add", stream=stream) for i in range(0, len(partial) - 1, 2)]
+        merged = [_run(Ewise(partial[i], partial[i + 1], "add", stream=stream), stats, stream)
+                  for i in range(0, len(partial) - 1, 2)]
         if len(partial) % 2:
             merged.append(partial[-1])
         partial = merged
