@@ -87,19 +87,31 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
   }
 }
 
+// Rows with at most kRcdCacheA stored A entries keep each entry's B-row
+// position, end and A value in shared memory (loaded once per row, in the
+// space of the cursors of longer rows); longer rows keep a cursor per entry
+// and reload the entry from global memory in every slice.
+constexpr int kRcdCacheA = 1024;
+
 template <typename T>
 __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const RowPlan<T> p, int width) {
+  static_assert(kRcdCacheA * (2 * sizeof(long long) + sizeof(T)) <= kRcdMaxA * sizeof(int),
+                "the entry cache shares the cursor space");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   T* dense = reinterpret_cast<T*>(smem_raw);                           // width values
   uint8_t* flags = smem_raw + static_cast<size_t>(width) * sizeof(T);  // width bytes
   int* a_cur = reinterpret_cast<int*>(flags + width);                  // kRcdMaxA cursors (offset in B row)
+  long long* c_pos = reinterpret_cast<long long*>(a_cur);              // or: kRcdCacheA positions in B,
+  long long* c_end = c_pos + kRcdCacheA;                               //     their row ends
+  T* c_av = reinterpret_cast<T*>(c_end + kRcdCacheA);                  //     and the A values
   __shared__ long long s_scan[32];
-  constexpr int kWarps = kRcdNumThreads / 32;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __shared__ int s_next;  // next stored A entry to hand out in the current slice
+  const int lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < width; i += kRcdNumThreads) {
     dense[i] = T(0);
     flags[i] = 0;
   }
+  if (threadIdx.x == 0) s_next = 0;
   __syncthreads();
   for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
     const int32_t row = p.perm[p.seg_begin + r];
@@ -109,39 +121,64 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
     const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);  // <= kRcdMaxA by classification
     const int64_t cbase = p.c_rowptr[row];
     const int64_t cend = p.c_rowptr[row + 1];
-    for (int j = threadIdx.x; j < na; j += kRcdNumThreads) a_cur[j] = 0;
+    const bool cached = na <= kRcdCacheA;
+    for (int j = threadIdx.x; j < na; j += kRcdNumThreads) {
+      if (cached) {
+        const int k = p.A.colidx[ra + j];
+        c_pos[j] = p.B.rowptr[k];
+        c_end[j] = p.B.rowptr[k + 1];
+        c_av[j] = p.A.vals[ra + j];
+      } else {
+        a_cur[j] = 0;
+      }
+    }
     __syncthreads();
     int64_t emitted = 0;
     bool bad = false;
     for (long long c0 = lo; c0 <= hi; c0 += width) {
       const long long c1 = min(c0 + width, static_cast<long long>(hi) + 1);
-      // Every warp walks the B rows of its stored A entries from their cursors,
-      // four loads in flight per lane; the columns of one B row are distinct,
-      // entries of different warps meet in shared-memory atomics.
-      for (int j = warp; j < na; j += kWarps) {
-        const int k = p.A.colidx[ra + j];
-        const T av = p.A.vals[ra + j];
-        const int64_t b0 = p.B.rowptr[k];
-        const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
-        int stop = len;
-        for (int t0 = a_cur[j]; t0 < len; t0 += 128) {
+      // Warps take stored A entries one at a time from a shared counter (long
+      // and short B rows balance out) and walk each B row from where the last
+      // slice stopped, four loads in flight per lane; the columns of one B row
+      // are distinct, entries of different warps meet in shared-memory atomics.
+      for (int guard = 0; guard <= na; ++guard) {
+        int j = 0;
+        if (lane == 0) j = atomicAdd(&s_next, 1);
+        j = __shfl_sync(kFull, j, 0);
+        if (j >= na) break;
+        long long b0, pos, end;
+        T av;
+        if (cached) {
+          pos = c_pos[j];
+          end = c_end[j];
+          av = c_av[j];
+          b0 = 0;
+        } else {
+          const int k = p.A.colidx[ra + j];
+          av = p.A.vals[ra + j];
+          b0 = p.B.rowptr[k];
+          end = p.B.rowptr[k + 1];
+          pos = b0 + a_cur[j];
+        }
+        long long stop = end;
+        for (long long t0 = pos; t0 < end; t0 += 128) {
           int cc[4];
           T bv[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int t = t0 + u * 32 + lane;
-            cc[u] = t < len ? p.B.colidx[b0 + t] : INT_MAX;
-            bv[u] = t < len ? p.B.vals[b0 + t] : T(0);
+            const long long t = t0 + u * 32 + lane;
+            cc[u] = t < end ? p.B.colidx[t] : INT_MAX;
+            bv[u] = t < end ? p.B.vals[t] : T(0);
           }
           bool past = false;
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int t = t0 + u * 32 + lane;
+            const long long t = t0 + u * 32 + lane;
             if (cc[u] < c1) {
               const int off = static_cast<int>(cc[u] - c0);
               atomicAdd(dense + off, av * bv[u]);
               flags[off] = 1;
-            } else if (t < len) {
+            } else if (t < end) {
               stop = min(stop, t);
               past = true;
             }
@@ -150,50 +187,53 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) stop = min(stop, __shfl_xor_sync(kFull, stop, o));
-        if (lane == 0) a_cur[j] = stop;
+        if (lane == 0) {
+          if (cached) {
+            c_pos[j] = stop;
+          } else {
+            a_cur[j] = static_cast<int>(stop - b0);
+          }
+        }
       }
       __syncthreads();
-      // Emit the slice in column order: warp w owns a contiguous block of
-      // 32-column chunks (at most 32), finds the touched ones with one 32-byte
-      // flag read per lane, and compacts them with ballots (coalesced stores).
+      // Emit the slice in column order: thread t owns the contiguous 16-byte
+      // flag chunks [t * cpt, (t + 1) * cpt); it counts their set flags, the
+      // CTA scans the counts, and every thread writes its entries in order
+      // and clears its chunks (work in proportion to the slice's columns / 16
+      // plus its entries).  Flags past the slice end are never set.
       const int w = static_cast<int>(c1 - c0);
-      const int nchunks = (w + 31) >> 5;
-      const int per_warp = (nchunks + kWarps - 1) / kWarps;
-      const int ch0 = warp * per_warp;
-      const int ch1 = min(ch0 + per_warp, nchunks);
-      bool touched = false;
-      if (ch0 + lane < ch1) {
-        const uint4* f4 = reinterpret_cast<const uint4*>(flags + ((ch0 + lane) << 5));
-        const uint4 x = f4[0], y = f4[1];
-        touched = (x.x | x.y | x.z | x.w | y.x | y.y | y.z | y.w) != 0u;
-      }
-      const unsigned tmask = __ballot_sync(kFull, touched);
+      const int nq = (w + 15) >> 4;
+      const int cpt = (nq + kRcdNumThreads - 1) / kRcdNumThreads;
+      const int q0 = threadIdx.x * cpt;
+      const int q1 = min(q0 + cpt, nq);
+      uint4* f4 = reinterpret_cast<uint4*>(flags);
       long long mine = 0;
-      for (unsigned tm = tmask; tm; tm &= tm - 1u) {
-        const int i = ((ch0 + __ffs(tm) - 1) << 5) + lane;
-        mine += __popc(__ballot_sync(kFull, i < w && flags[i] != 0));
-      }
+      for (int q = q0; q < q1; ++q) mine += nonzero_bytes(f4[q]);
       long long total;
-      const long long ex = block_exclusive_scan(lane == 0 ? mine : 0ll, s_scan, &total);
-      int64_t pos = cbase + emitted + __shfl_sync(kFull, ex, 0);
-      for (unsigned tm = tmask; tm; tm &= tm - 1u) {
-        const int i = ((ch0 + __ffs(tm) - 1) << 5) + lane;
-        const bool f = i < w && flags[i] != 0;
-        const unsigned m = __ballot_sync(kFull, f);
-        if (f) {
-          const int64_t q = pos + __popc(m & ((1u << lane) - 1u));
-          if (q < cend) {
-            p.c_colidx[q] = static_cast<int32_t>(c0 + i);
-            p.c_vals[q] = dense[i];
-          } else {
-            bad = true;
+      const long long before = block_exclusive_scan(mine, s_scan, &total);
+      int64_t pos = cbase + emitted + before;
+      for (int q = q0; q < q1; ++q) {
+        const uint4 v = f4[q];
+        const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          // bytes of this word that are set, lowest column first
+          for (uint32_t m = __vcmpne4(words[h], 0u) & 0x01010101u; m; m &= m - 1u) {
+            const int i = (q << 4) + (h << 2) + ((__ffs(m) - 1) >> 3);
+            if (pos < cend) {
+              p.c_colidx[pos] = static_cast<int32_t>(c0 + i);
+              p.c_vals[pos] = dense[i];
+            } else {
+              bad = true;
+            }
+            dense[i] = T(0);
+            ++pos;
           }
-          flags[i] = 0;
-          dense[i] = T(0);
         }
-        pos += __popc(m);
+        f4[q] = make_uint4(0u, 0u, 0u, 0u);
       }
       emitted += total;
+      if (threadIdx.x == 0) s_next = 0;  // every warp has left this slice's entry loop
       __syncthreads();
     }
     if (threadIdx.x == 0 && emitted != cend - cbase) bad = true;
