@@ -96,6 +96,7 @@ struct Plan {
   DevBuf ranks;   // register bitmap rows: kBmrSlots uint16 ranks per row of A
   DevBuf ew;      // elementwise operations: summary, chunk arrays, scan partials
   DevBuf sv;      // sparse matrix - sparse vector product (in A^T's handle): accumulator, byte-map, offsets
+  DevBuf rcd;     // dense heavy rows: per-slice counts, mega-row list, work counters
   int kind = kPlanNone;  // which symbolic pass filled this plan
   // elementwise plan (kPlanEwise)
   int ew_op = 0, ew_group = 32;
@@ -104,6 +105,10 @@ struct Plan {
   int32_t* ew_chunk_row = nullptr;
   int64_t* ew_chunk_off = nullptr;
   int64_t* ew_partials = nullptr;
+  int32_t* rcd_scnt = nullptr;
+  int32_t* rcd_mega = nullptr;
+  int32_t* rcd_nmega = nullptr;
+  int32_t* rcd_ctr = nullptr;
   // submatrix plan (kPlanSub): the block the symbolic pass counted
   int64_t sub_r0 = 0, sub_r1 = 0, sub_c0 = 0, sub_c1 = 0;
   DevSummary* host_sum = nullptr;  // pinned
@@ -277,8 +282,24 @@ ws_status_t symbolic_bins(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
     launch_dense<T>(p, pl->dense_slices, false, sms, s, &pl->sym_launches);
   }
   if (pl->seg_count[kSegRcd] > 0) {
+    const int64_t nr = pl->seg_count[kSegRcd];
+    const size_t o_scnt = 0;
+    const size_t o_mega = align_up(o_scnt + 4 * static_cast<size_t>(nr) * rcd_slices<T>(), 256);
+    const size_t o_cnt = align_up(o_mega + 4 * static_cast<size_t>(nr), 256);
+    st = pl->rcd.reserve(o_cnt + 256, s);
+    if (st != WS_OK) return st;
+    char* b = static_cast<char*>(pl->rcd.ptr);
+    pl->rcd_scnt = reinterpret_cast<int32_t*>(b + o_scnt);
+    pl->rcd_mega = reinterpret_cast<int32_t*>(b + o_mega);
+    pl->rcd_nmega = reinterpret_cast<int32_t*>(b + o_cnt);
+    pl->rcd_ctr = pl->rcd_nmega + 1;
+    WS_CUDA(cudaMemsetAsync(pl->rcd_nmega, 0, sizeof(int32_t), s), "cudaMemsetAsync(rcd counters)");
+    p.rcd_scnt = pl->rcd_scnt;
+    p.rcd_mega = pl->rcd_mega;
+    p.rcd_nmega = pl->rcd_nmega;
+    p.rcd_ctr = pl->rcd_ctr;
     p.seg_begin = pl->seg_offset[kSegRcd];
-    p.seg_len = pl->seg_count[kSegRcd];
+    p.seg_len = nr;
     launch_rcd<T>(p, false, sms, s, &pl->sym_launches);
   }
   if (pl->seg_count[kSegWb] > 0) {
@@ -406,6 +427,11 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     p.perm = pl->perm;
   }
   if (pl->seg_count[kSegRcd] > 0) {
+    WS_CUDA(cudaMemsetAsync(pl->rcd_ctr, 0, 2 * sizeof(int32_t), s), "cudaMemsetAsync(rcd work counters)");
+    p.rcd_scnt = pl->rcd_scnt;
+    p.rcd_mega = pl->rcd_mega;
+    p.rcd_nmega = pl->rcd_nmega;
+    p.rcd_ctr = pl->rcd_ctr;
     p.seg_begin = pl->seg_offset[kSegRcd];
     p.seg_len = pl->seg_count[kSegRcd];
     launch_rcd<T>(p, true, sms, s, &pl->num_launches);
@@ -895,13 +921,15 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream) {
 ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
-    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr || h->plan->sv.ptr)
+    if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr || h->plan->sv.ptr ||
+        h->plan->rcd.ptr)
       cudaDeviceSynchronize();
     h->plan->rows.release();
     h->plan->slices.release();
     h->plan->ranks.release();
     h->plan->ew.release();
     h->plan->sv.release();
+    h->plan->rcd.release();
     if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
     delete h->plan;
   }

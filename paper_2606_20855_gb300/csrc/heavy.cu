@@ -39,6 +39,12 @@ constexpr int kWbThreads = 512;
 
 // ---------------------------------------------------------------- dense rows
 
+constexpr int kRcdCacheA = 1024;  // stored A entries of a row kept in shared memory (and of a batch)
+// Rows with more stored A entries are split into (row, slice) items (256 was
+// faster than 64 or 1024 on the R-MAT inputs; splitting every row was 1.8x slower).
+constexpr int kRcdMegaA = 256;
+static_assert(kRcdMegaA <= kRcdCacheA, "rows done whole keep all entries in shared memory");
+
 // Counts the non-zero bytes of 16 bytes.
 __device__ __forceinline__ int nonzero_bytes(const uint4 v) {
   return __popc(__vcmpne4(v.x, 0u) & 0x01010101u) + __popc(__vcmpne4(v.y, 0u) & 0x01010101u) +
@@ -51,9 +57,12 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
   uint8_t* flags = smem_raw;  // kMaxBitmapSpan bytes
   uint4* flags4 = reinterpret_cast<uint4*>(smem_raw);
   __shared__ long long s_scan[32];
+  constexpr int kS = rcd_slices<T>();
+  __shared__ int s_slice[kS];  // entries per dense-window slice of the row
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr int kWarps = kRcdThreads / 32;
   for (int i = threadIdx.x; i < kMaxBitmapSpan / 16; i += kRcdThreads) flags4[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (threadIdx.x < kS) s_slice[threadIdx.x] = 0;
   __syncthreads();
   for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
     const int32_t row = p.perm[p.seg_begin + r];
@@ -76,90 +85,256 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
     __syncthreads();
     long long cnt = 0;
     const int n16 = (span + 15) >> 4;
+    constexpr int kChunksPerSlice = kRcdWidthBytes / static_cast<int>(sizeof(T)) / 16;
     for (int i = threadIdx.x; i < n16; i += kRcdThreads) {
-      cnt += nonzero_bytes(flags4[i]);
+      const int n = nonzero_bytes(flags4[i]);
+      cnt += n;
+      if (n) atomicAdd(&s_slice[i / kChunksPerSlice], n);
       flags4[i] = make_uint4(0u, 0u, 0u, 0u);
     }
     long long total;
     block_exclusive_scan(cnt, s_scan, &total);
-    if (threadIdx.x == 0) p.c_rowptr[row + 1] = total;
+    if (threadIdx.x == 0) {
+      p.c_rowptr[row + 1] = total;
+      if (re - ra > kRcdMegaA) p.rcd_mega[atomicAdd(p.rcd_nmega, 1)] = static_cast<int32_t>(r);
+    }
+    if (threadIdx.x < kS) {
+      p.rcd_scnt[r * kS + threadIdx.x] = s_slice[threadIdx.x];
+      s_slice[threadIdx.x] = 0;
+    }
     __syncthreads();
   }
 }
 
-// Rows with at most kRcdCacheA stored A entries keep each entry's B-row
-// position, end and A value in shared memory (loaded once per row, in the
-// space of the cursors of longer rows); longer rows keep a cursor per entry
-// and reload the entry from global memory in every slice.
-constexpr int kRcdCacheA = 1024;
+// Numeric pass of the dense heavy rows.  Two kinds of work, taken from two
+// counters so CTAs balance themselves:
+//   1. mega rows (more than kRcdMegaA stored A entries, typically the hub
+//      rows of a power-law matrix): every (row, slice) pair is a separate
+//      item, so one row's slices run on several CTAs at once.  An item finds
+//      the part of each entry's B row inside its slice by binary search
+//      (one lane per entry, kRcdBatch entries at a time), walks the long
+//      parts with a warp each and the short ones with a lane each, and emits
+//      the slice from the offset the symbolic pass's per-slice counts give.
+//   2. the other rows: one CTA per row, slices in order; each entry's B-row
+//      position, end and A value stay in shared memory for the whole row and
+//      every slice continues where the last one stopped.
+constexpr int kRcdShort = 32;  // parts of B rows walked by a single lane
+
+// Emits one slice of the dense window in column order: thread t owns the
+// contiguous 16-byte flag chunks [t * cpt, (t + 1) * cpt); it counts their set
+// flags, the CTA scans the counts, and every thread writes its entries in
+// order from `pos0` and clears its chunks and values.  Returns the count.
+template <typename T>
+__device__ long long rcd_emit(const RowPlan<T>& p, T* dense, uint8_t* flags, int w, long long c0, int64_t pos0,
+                              int64_t cend, long long* s_scan, bool* bad) {
+  const int nq = (w + 15) >> 4;
+  const int cpt = (nq + kRcdNumThreads - 1) / kRcdNumThreads;
+  const int q0 = threadIdx.x * cpt;
+  const int q1 = min(q0 + cpt, nq);
+  uint4* f4 = reinterpret_cast<uint4*>(flags);
+  long long mine = 0;
+  for (int q = q0; q < q1; ++q) mine += nonzero_bytes(f4[q]);
+  long long total;
+  const long long before = block_exclusive_scan(mine, s_scan, &total);
+  int64_t pos = pos0 + before;
+  for (int q = q0; q < q1; ++q) {
+    const uint4 v = f4[q];
+    const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      // bytes of this word that are set, lowest column first
+      for (uint32_t m = __vcmpne4(words[h], 0u) & 0x01010101u; m; m &= m - 1u) {
+        const int i = (q << 4) + (h << 2) + ((__ffs(m) - 1) >> 3);
+        if (pos < cend) {
+          p.c_colidx[pos] = static_cast<int32_t>(c0 + i);
+          p.c_vals[pos] = dense[i];
+        } else {
+          *bad = true;
+        }
+        dense[i] = T(0);
+        ++pos;
+      }
+    }
+    f4[q] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  return total;
+}
+
+// Adds a * B[., c] for the B entries [b, b + n) (all inside [c0, c1)) into the
+// window, a warp at a time, four loads in flight per lane.
+template <typename T>
+__device__ __forceinline__ void rcd_warp_add(const RowPlan<T>& p, T* dense, uint8_t* flags, long long b, long long n,
+                                             T av, long long c0, int lane) {
+  for (long long t0 = 0; t0 < n; t0 += 128) {
+    int cc[4];
+    T bv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long t = t0 + u * 32 + lane;
+      cc[u] = t < n ? p.B.colidx[b + t] : -1;
+      bv[u] = t < n ? p.B.vals[b + t] : T(0);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (cc[u] >= 0) {
+        const int off = static_cast<int>(cc[u] - c0);
+        atomicAdd(dense + off, av * bv[u]);
+        flags[off] = 1;
+      }
+    }
+  }
+}
+
+// First position in cols[0..n) with cols[pos] >= c (n if none).
+__device__ __forceinline__ long long first_at_least(const int32_t* cols, long long n, long long c) {
+  long long lo = 0, hi = n;
+  while (lo < hi) {  // O(log n) probes
+    const long long mid = (lo + hi) >> 1;
+    if (cols[mid] < c) {
+      lo = mid + 1;
+    } else {
+      hi = mid;
+    }
+  }
+  return lo;
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const RowPlan<T> p, int width) {
-  static_assert(kRcdCacheA * (2 * sizeof(long long) + sizeof(T)) <= kRcdMaxA * sizeof(int),
-                "the entry cache shares the cursor space");
+  constexpr int kS = rcd_slices<T>();
+  static_assert(kRcdCacheA * (2 * sizeof(long long) + sizeof(T) + sizeof(int)) <= kRcdMaxA * sizeof(int),
+                "the entry cache fits the space after the window");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   T* dense = reinterpret_cast<T*>(smem_raw);                           // width values
   uint8_t* flags = smem_raw + static_cast<size_t>(width) * sizeof(T);  // width bytes
-  int* a_cur = reinterpret_cast<int*>(flags + width);                  // kRcdMaxA cursors (offset in B row)
-  long long* c_pos = reinterpret_cast<long long*>(a_cur);              // or: kRcdCacheA positions in B,
-  long long* c_end = c_pos + kRcdCacheA;                               //     their row ends
-  T* c_av = reinterpret_cast<T*>(c_end + kRcdCacheA);                  //     and the A values
+  long long* c_pos = reinterpret_cast<long long*>(flags + width);      // per entry: position in B,
+  long long* c_end = c_pos + kRcdCacheA;                               //   end of the B row (or of the part),
+  T* c_av = reinterpret_cast<T*>(c_end + kRcdCacheA);                  //   the A value,
+  int* c_long = reinterpret_cast<int*>(c_av + kRcdCacheA);             //   and the list of long parts
   __shared__ long long s_scan[32];
-  __shared__ int s_next;  // next stored A entry to hand out in the current slice
+  __shared__ int s_item, s_next, s_next2, s_nlong;
+  __shared__ long long s_out0;
   const int lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < width; i += kRcdNumThreads) {
     dense[i] = T(0);
     flags[i] = 0;
   }
-  if (threadIdx.x == 0) s_next = 0;
-  __syncthreads();
-  for (int64_t r = blockIdx.x; r < p.seg_len; r += gridDim.x) {
+  bool bad = false;
+  const int n_mega = *p.rcd_nmega;
+
+  // 1. (mega row, slice) items
+  for (int guard = 0; guard <= n_mega * kS; ++guard) {
+    __syncthreads();  // the previous item is done with the shared state
+    if (threadIdx.x == 0) {
+      s_item = atomicAdd(p.rcd_ctr, 1);
+      s_nlong = 0;
+    }
+    __syncthreads();
+    const int item = s_item;
+    if (item >= n_mega * kS) break;
+    const int r = p.rcd_mega[item / kS], sl = item % kS;
     const int32_t row = p.perm[p.seg_begin + r];
-    const int lo = p.lo[row];
-    const int hi = p.hi[row];
+    const long long lo = p.lo[row], hi = p.hi[row];
+    const long long c0 = lo + static_cast<long long>(sl) * width;
+    if (c0 > hi) continue;
+    const long long c1 = min(c0 + width, hi + 1);
+    if (threadIdx.x == 0) {
+      long long o = p.c_rowptr[row];
+      for (int t = 0; t < sl; ++t) o += p.rcd_scnt[static_cast<int64_t>(r) * kS + t];
+      s_out0 = o;
+    }
     const int64_t ra = p.A.rowptr[row];
-    const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);  // <= kRcdMaxA by classification
+    const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
+    for (int e0 = 0; e0 < na; e0 += kRcdCacheA) {
+      const int nb = min(kRcdCacheA, na - e0);
+      for (int j = threadIdx.x; j < nb; j += kRcdNumThreads) {
+        const int k = p.A.colidx[ra + e0 + j];
+        const long long b0 = p.B.rowptr[k], len = p.B.rowptr[k + 1] - b0;
+        const long long st = first_at_least(p.B.colidx + b0, len, c0);
+        const long long en = st + first_at_least(p.B.colidx + b0 + st, len - st, c1);
+        c_pos[j] = b0 + st;
+        c_end[j] = b0 + en;
+        c_av[j] = p.A.vals[ra + e0 + j];
+        if (en - st > kRcdShort) c_long[atomicAdd(&s_nlong, 1)] = j;
+      }
+      if (threadIdx.x == 0) {
+        s_next = 0;
+        s_next2 = 0;
+      }
+      __syncthreads();
+      const int nl = s_nlong;
+      for (int g2 = 0; g2 <= nl; ++g2) {  // long parts: a warp each
+        int t = 0;
+        if (lane == 0) t = atomicAdd(&s_next, 1);
+        t = __shfl_sync(kFull, t, 0);
+        if (t >= nl) break;
+        const int j = c_long[t];
+        rcd_warp_add(p, dense, flags, c_pos[j], c_end[j] - c_pos[j], c_av[j], c0, lane);
+      }
+      for (int g2 = 0; g2 <= nb / 32 + 1; ++g2) {  // short parts: a lane each
+        int base = 0;
+        if (lane == 0) base = atomicAdd(&s_next2, 32);
+        base = __shfl_sync(kFull, base, 0);
+        if (base >= nb) break;
+        const int j = base + lane;
+        if (j < nb && c_end[j] - c_pos[j] <= kRcdShort) {
+          const T av = c_av[j];
+          for (long long t = c_pos[j]; t < c_end[j]; ++t) {
+            const int off = static_cast<int>(p.B.colidx[t] - c0);
+            atomicAdd(dense + off, av * p.B.vals[t]);
+            flags[off] = 1;
+          }
+        }
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) s_nlong = 0;
+      __syncthreads();
+    }
+    const int64_t want = p.rcd_scnt[static_cast<int64_t>(r) * kS + sl];
+    const long long got = rcd_emit(p, dense, flags, static_cast<int>(c1 - c0), c0, s_out0, s_out0 + want, s_scan, &bad);
+    if (threadIdx.x == 0 && got != want) bad = true;
+  }
+
+  // 2. the other rows, one CTA each
+  for (int guard = 0; guard <= p.seg_len; ++guard) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s_item = atomicAdd(p.rcd_ctr + 1, 1);
+      s_nlong = 0;
+      s_next = 0;
+      s_next2 = 0;
+    }
+    __syncthreads();
+    const int r = s_item;
+    if (r >= p.seg_len) break;
+    const int32_t row = p.perm[p.seg_begin + r];
+    const int64_t ra = p.A.rowptr[row];
+    const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
+    if (na > kRcdMegaA) continue;  // a mega row: done in part 1
+    const long long lo = p.lo[row], hi = p.hi[row];
     const int64_t cbase = p.c_rowptr[row];
     const int64_t cend = p.c_rowptr[row + 1];
-    const bool cached = na <= kRcdCacheA;
     for (int j = threadIdx.x; j < na; j += kRcdNumThreads) {
-      if (cached) {
-        const int k = p.A.colidx[ra + j];
-        c_pos[j] = p.B.rowptr[k];
-        c_end[j] = p.B.rowptr[k + 1];
-        c_av[j] = p.A.vals[ra + j];
-      } else {
-        a_cur[j] = 0;
-      }
+      const int k = p.A.colidx[ra + j];
+      c_pos[j] = p.B.rowptr[k];
+      c_end[j] = p.B.rowptr[k + 1];
+      c_av[j] = p.A.vals[ra + j];
     }
     __syncthreads();
     int64_t emitted = 0;
-    bool bad = false;
     for (long long c0 = lo; c0 <= hi; c0 += width) {
-      const long long c1 = min(c0 + width, static_cast<long long>(hi) + 1);
-      // Warps take stored A entries one at a time from a shared counter (long
-      // and short B rows balance out) and walk each B row from where the last
-      // slice stopped, four loads in flight per lane; the columns of one B row
-      // are distinct, entries of different warps meet in shared-memory atomics.
-      for (int guard = 0; guard <= na; ++guard) {
+      const long long c1 = min(c0 + width, hi + 1);
+      // Warps take stored A entries one at a time from a shared counter and
+      // walk each B row from where the last slice stopped, four loads in
+      // flight per lane; the columns of one B row are distinct, entries of
+      // different warps meet in shared-memory atomics.
+      for (int g2 = 0; g2 <= na; ++g2) {
         int j = 0;
         if (lane == 0) j = atomicAdd(&s_next, 1);
         j = __shfl_sync(kFull, j, 0);
         if (j >= na) break;
-        long long b0, pos, end;
-        T av;
-        if (cached) {
-          pos = c_pos[j];
-          end = c_end[j];
-          av = c_av[j];
-          b0 = 0;
-        } else {
-          const int k = p.A.colidx[ra + j];
-          av = p.A.vals[ra + j];
-          b0 = p.B.rowptr[k];
-          end = p.B.rowptr[k + 1];
-          pos = b0 + a_cur[j];
-        }
+        const long long pos = c_pos[j], end = c_end[j];
+        const T av = c_av[j];
         long long stop = end;
         for (long long t0 = pos; t0 < end; t0 += 128) {
           int cc[4];
@@ -187,58 +362,16 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) stop = min(stop, __shfl_xor_sync(kFull, stop, o));
-        if (lane == 0) {
-          if (cached) {
-            c_pos[j] = stop;
-          } else {
-            a_cur[j] = static_cast<int>(stop - b0);
-          }
-        }
+        if (lane == 0) c_pos[j] = stop;
       }
       __syncthreads();
-      // Emit the slice in column order: thread t owns the contiguous 16-byte
-      // flag chunks [t * cpt, (t + 1) * cpt); it counts their set flags, the
-      // CTA scans the counts, and every thread writes its entries in order
-      // and clears its chunks (work in proportion to the slice's columns / 16
-      // plus its entries).  Flags past the slice end are never set.
-      const int w = static_cast<int>(c1 - c0);
-      const int nq = (w + 15) >> 4;
-      const int cpt = (nq + kRcdNumThreads - 1) / kRcdNumThreads;
-      const int q0 = threadIdx.x * cpt;
-      const int q1 = min(q0 + cpt, nq);
-      uint4* f4 = reinterpret_cast<uint4*>(flags);
-      long long mine = 0;
-      for (int q = q0; q < q1; ++q) mine += nonzero_bytes(f4[q]);
-      long long total;
-      const long long before = block_exclusive_scan(mine, s_scan, &total);
-      int64_t pos = cbase + emitted + before;
-      for (int q = q0; q < q1; ++q) {
-        const uint4 v = f4[q];
-        const uint32_t words[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          // bytes of this word that are set, lowest column first
-          for (uint32_t m = __vcmpne4(words[h], 0u) & 0x01010101u; m; m &= m - 1u) {
-            const int i = (q << 4) + (h << 2) + ((__ffs(m) - 1) >> 3);
-            if (pos < cend) {
-              p.c_colidx[pos] = static_cast<int32_t>(c0 + i);
-              p.c_vals[pos] = dense[i];
-            } else {
-              bad = true;
-            }
-            dense[i] = T(0);
-            ++pos;
-          }
-        }
-        f4[q] = make_uint4(0u, 0u, 0u, 0u);
-      }
-      emitted += total;
+      emitted += rcd_emit(p, dense, flags, static_cast<int>(c1 - c0), c0, cbase + emitted, cend, s_scan, &bad);
       if (threadIdx.x == 0) s_next = 0;  // every warp has left this slice's entry loop
       __syncthreads();
     }
     if (threadIdx.x == 0 && emitted != cend - cbase) bad = true;
-    if (bad) atomicOr(&p.sum->status, kErrCount);
   }
+  if (bad) atomicOr(&p.sum->status, kErrCount);
 }
 
 // ----------------------------------------------------------------- wide rows
@@ -368,7 +501,8 @@ int grid_of(int64_t rows, int num_sms, int per_sm) {
 }  // namespace
 
 size_t rcd_numeric_smem(int width, size_t value_bytes) {
-  return static_cast<size_t>(width) * (value_bytes + 1) + static_cast<size_t>(kRcdMaxA) * 4;
+  return static_cast<size_t>(width) * (value_bytes + 1) +
+         static_cast<size_t>(kRcdCacheA) * (2 * sizeof(long long) + value_bytes + sizeof(int));
 }
 
 template <typename T>

@@ -75,6 +75,11 @@ constexpr uint8_t kClsWb = kClsRcd + 1;         // heavy rows, wide bitmap works
 constexpr int kRcdMaxA = 8192;            // stored A entries a dense row may have (cursor slots)
 constexpr int kRcdDefaultMaxA = 8192;     // default limit used by the classification
 constexpr int kRcdWidthBytes = 65536;     // dense value window per slice
+// Dense-window slices of a dense heavy row (its span is at most kMaxBitmapSpan columns).
+template <typename T>
+constexpr int rcd_slices() {
+  return (kMaxBitmapSpan + kRcdWidthBytes / static_cast<int>(sizeof(T)) - 1) / (kRcdWidthBytes / static_cast<int>(sizeof(T)));
+}
 constexpr int kWbMaxSpan = 1 << 20;       // widest column range of a wide-bitmap row
 
 // Segments of the row permutation: direct rows, register bitmap bins, bitmap
@@ -140,6 +145,10 @@ struct RowPlan {
   const int32_t* slice_first;
   int32_t* slice_cnt;          // entries per dense-window slice
   uint16_t* ranks;             // register bitmap rows: output position of every product, kBmrSlots per row
+  int32_t* rcd_scnt;           // dense heavy rows: entries per dense-window slice, rcd_slices<T>() per row
+  int32_t* rcd_mega;           // dense heavy rows with more than 1024 stored A entries (segment positions)
+  int32_t* rcd_nmega;          // their number
+  int32_t* rcd_ctr;            // two work counters of the numeric kernel (zeroed before it)
   DevSummary* sum;
   int64_t seg_begin;   // first position in perm of the segment a kernel processes
   int64_t seg_len;     // rows in that segment
