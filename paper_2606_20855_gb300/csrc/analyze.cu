@@ -155,13 +155,18 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
 }
 
-// One warp per long row; lanes stride over the row's stored entries.
+// One CTA per long row (a power-law row can hold tens of thousands of
+// entries, and its three dependent loads per entry are a latency chain):
+// threads stride over the row's stored entries, eight in flight each, and
+// the CTA reduces the product count and column range.
 template <typename T>
 __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, const AnalyzeParams ap,
                                                            const int32_t* long_rows) {
   __shared__ int s_seg[kNumSegs];
   __shared__ long long s_prod, s_slices;
   __shared__ int s_empty;
+  __shared__ long long s_ub[8];
+  __shared__ int s_lo[8], s_hi[8];
   if (threadIdx.x < kNumSegs) s_seg[threadIdx.x] = 0;
   if (threadIdx.x == 0) {
     s_prod = 0;
@@ -169,17 +174,15 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
     s_empty = 0;
   }
   __syncthreads();
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nlong = *reinterpret_cast<volatile int*>(&p.sum->n_long);
-  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
-  for (int64_t w = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); w < nlong;
-       w += warps) {
+  for (int64_t w = blockIdx.x; w < nlong; w += gridDim.x) {
     const int64_t i = long_rows[w];
     const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
     long long ub = 0;
     int lo = INT_MAX, hi = -1;
-#pragma unroll 4
-    for (int64_t q = s + lane; q < e; q += 32) {
+#pragma unroll 8
+    for (int64_t q = s + threadIdx.x; q < e; q += blockDim.x) {
       const int k = p.A.colidx[q];
       const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];
       if (be > bs) {
@@ -194,7 +197,21 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
       lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
       hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
-    if (lane == 0) record_row(p, ap, i, e - s, ub, lo, hi, INT_MAX, s_seg, &s_prod, &s_slices, &s_empty);
+    if (lane == 0) {
+      s_ub[warp] = ub;
+      s_lo[warp] = lo;
+      s_hi[warp] = hi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      for (int w2 = 1; w2 < static_cast<int>(blockDim.x >> 5); ++w2) {
+        ub += s_ub[w2];
+        lo = min(lo, s_lo[w2]);
+        hi = max(hi, s_hi[w2]);
+      }
+      record_row(p, ap, i, e - s, ub, lo, hi, INT_MAX, s_seg, &s_prod, &s_slices, &s_empty);
+    }
+    __syncthreads();  // s_ub/s_lo/s_hi are reused by the next row
   }
   __syncthreads();
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
@@ -291,7 +308,7 @@ template <typename T>
 void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, const int32_t* rows,
                     int num_sms, cudaStream_t s, int* launches) {
   analyze_kernel<T><<<grid_for(ap.m, 256, num_sms, 8), 256, 0, s>>>(p, ap, long_rows, rows);
-  analyze_long_kernel<T><<<num_sms * 2, 256, 0, s>>>(p, ap, long_rows);
+  analyze_long_kernel<T><<<num_sms * 4, 256, 0, s>>>(p, ap, long_rows);
   *launches += 2;
 }
 

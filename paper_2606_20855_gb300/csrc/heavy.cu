@@ -36,6 +36,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kRcdThreads = 256;
 constexpr int kRcdNumThreads = 512;
 constexpr int kWbThreads = 512;
+constexpr int kWbBatch = 4;  // stored A entries a lane group has in flight in the wide-bitmap kernel
 
 // ---------------------------------------------------------------- dense rows
 
@@ -402,18 +403,33 @@ __global__ void __launch_bounds__(kWbThreads, 1) wb_kernel(const RowPlan<T> p) {
       cend = p.c_rowptr[row + 1];
       for (int64_t i = cbase + threadIdx.x; i < cend; i += kWbThreads) p.c_vals[i] = T(0);
     }
-    // Set the bit of every product column.
+    // Set the bit of every product column.  A group takes kWbBatch stored A
+    // entries per round, so their row-pointer and column loads are in flight
+    // together (a hub row has tens of thousands of entries).
     long long fresh = 0;
-    for (int64_t pa = ra + grp; pa < re; pa += ngrp) {
-      const int k = p.A.colidx[pa];
-      const int64_t qe = p.B.rowptr[k + 1];
-      for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
-        const uint32_t off = static_cast<uint32_t>(p.B.colidx[q] - lo);
-        const uint32_t bit = 1u << (off & 31u);
-        if constexpr (NUMERIC) {
-          atomicOr(bm + (off >> 5), bit);
-        } else {
-          fresh += (atomicOr(bm + (off >> 5), bit) & bit) == 0u;
+    for (int64_t pa0 = ra + grp; pa0 < re; pa0 += static_cast<int64_t>(kWbBatch) * ngrp) {
+      int64_t qb[kWbBatch], qe[kWbBatch];
+#pragma unroll
+      for (int u = 0; u < kWbBatch; ++u) {
+        const int64_t pa = pa0 + static_cast<int64_t>(u) * ngrp;
+        qb[u] = 0;
+        qe[u] = 0;
+        if (pa < re) {
+          const int k = p.A.colidx[pa];
+          qb[u] = p.B.rowptr[k];
+          qe[u] = p.B.rowptr[k + 1];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kWbBatch; ++u) {
+        for (int64_t q = qb[u] + gl; q < qe[u]; q += gsize) {
+          const uint32_t off = static_cast<uint32_t>(p.B.colidx[q] - lo);
+          const uint32_t bit = 1u << (off & 31u);
+          if constexpr (NUMERIC) {
+            atomicOr(bm + (off >> 5), bit);
+          } else {
+            fresh += (atomicOr(bm + (off >> 5), bit) & bit) == 0u;
+          }
         }
       }
     }
@@ -455,11 +471,26 @@ __global__ void __launch_bounds__(kWbThreads, 1) wb_kernel(const RowPlan<T> p) {
         }
       }
       __syncthreads();  // prefixes and the zeroed values are visible to the CTA
-      for (int64_t pa = ra + grp; pa < re; pa += ngrp) {
-        const int k = p.A.colidx[pa];
-        const T av = p.A.vals[pa];
-        const int64_t qe = p.B.rowptr[k + 1];
-        for (int64_t q = p.B.rowptr[k] + gl; q < qe; q += gsize) {
+      for (int64_t pa0 = ra + grp; pa0 < re; pa0 += static_cast<int64_t>(kWbBatch) * ngrp) {
+        int64_t qb[kWbBatch], qe[kWbBatch];
+        T avs[kWbBatch];
+#pragma unroll
+        for (int u = 0; u < kWbBatch; ++u) {
+          const int64_t pa = pa0 + static_cast<int64_t>(u) * ngrp;
+          qb[u] = 0;
+          qe[u] = 0;
+          avs[u] = T(0);
+          if (pa < re) {
+            const int k = p.A.colidx[pa];
+            avs[u] = p.A.vals[pa];
+            qb[u] = p.B.rowptr[k];
+            qe[u] = p.B.rowptr[k + 1];
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kWbBatch; ++u) {
+        const T av = avs[u];
+        for (int64_t q = qb[u] + gl; q < qe[u]; q += gsize) {
           const uint32_t off = static_cast<uint32_t>(p.B.colidx[q] - lo);
           const uint32_t i = off >> 7;
           const uint4 v = bm4[i];
@@ -472,6 +503,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) wb_kernel(const RowPlan<T> p) {
           } else {
             bad = true;
           }
+        }
         }
       }
       if (bad) atomicOr(&p.sum->status, kErrCount);
