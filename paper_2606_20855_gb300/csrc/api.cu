@@ -15,6 +15,7 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <vector>
 
 #include "ws_internal.cuh"
 #include "ws_spgemm.h"
@@ -81,12 +82,58 @@ struct DevBuf {
     bytes = want;
     return WS_OK;
   }
+  // Returns the memory to the stream-ordered pool (callers synchronise the
+  // device first, so no queued work still uses it).
   void release() {
-    if (ptr) cudaFree(ptr);
+    if (ptr) cudaFreeAsync(ptr, nullptr);
     ptr = nullptr;
     bytes = 0;
   }
 };
+
+// Pinned host copies of the summary block, recycled across handles: a
+// cudaMallocHost / cudaFreeHost pair per handle costs more than a small
+// product.  Blocks are allocated 64 at a time and kept until the process
+// exits.
+std::mutex g_host_sum_mutex;
+std::vector<DevSummary*> g_host_sum_free;
+
+DevSummary* acquire_host_sum() {
+  std::lock_guard<std::mutex> lock(g_host_sum_mutex);
+  if (g_host_sum_free.empty()) {
+    constexpr int kBlocks = 64;
+    const size_t each = (sizeof(DevSummary) + 255) / 256 * 256;
+    char* base = nullptr;
+    if (cudaMallocHost(reinterpret_cast<void**>(&base), each * kBlocks) != cudaSuccess) return nullptr;
+    for (int i = kBlocks - 1; i >= 0; --i) g_host_sum_free.push_back(reinterpret_cast<DevSummary*>(base + i * each));
+  }
+  DevSummary* h = g_host_sum_free.back();
+  g_host_sum_free.pop_back();
+  return h;
+}
+
+void release_host_sum(DevSummary* h) {
+  if (!h) return;
+  std::lock_guard<std::mutex> lock(g_host_sum_mutex);
+  g_host_sum_free.push_back(h);
+}
+
+// Once per device: let the default stream-ordered pool keep freed memory
+// (its default releases it to the system at every synchronisation, so the
+// next handle's scratch would be allocated from scratch again).  This is a
+// setting of this process's pool, not of the GPU.
+void keep_pool_memory(int dev) {
+  static std::mutex m;
+  static bool done[64] = {};
+  std::lock_guard<std::mutex> lock(m);
+  if (dev < 0 || dev >= 64 || done[dev]) return;
+  cudaMemPool_t pool;
+  if (cudaDeviceGetDefaultMemPool(&pool, dev) == cudaSuccess) {
+    uint64_t keep = UINT64_MAX;
+    cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+  }
+  done[dev] = true;
+}
 
 enum PlanKind { kPlanNone = 0, kPlanSpgemm = 1, kPlanEwise = 2, kPlanSub = 3 };
 
@@ -570,11 +617,9 @@ ws_status_t ensure_plan(ws_csr_s* h) {
     if (!h->plan) return fail(WS_ERR_ALLOC, "host allocation failed");
   }
   if (!h->plan->host_sum) {
-    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&h->plan->host_sum), sizeof(DevSummary));
-    if (e != cudaSuccess) {
-      h->plan->host_sum = nullptr;
-      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
-    }
+    keep_pool_memory(h->device);
+    h->plan->host_sum = acquire_host_sum();
+    if (!h->plan->host_sum) return fail(WS_ERR_ALLOC, "cudaMallocHost failed");
   }
   return WS_OK;
 }
@@ -645,11 +690,9 @@ ws_status_t prepare_output(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C) {
   }
   Plan* pl = C->plan;
   if (!pl->host_sum) {
-    cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&pl->host_sum), sizeof(DevSummary));
-    if (e != cudaSuccess) {
-      pl->host_sum = nullptr;
-      return fail(WS_ERR_ALLOC, "cudaMallocHost: %s", cudaGetErrorString(e));
-    }
+    keep_pool_memory(C->device);
+    pl->host_sum = acquire_host_sum();
+    if (!pl->host_sum) return fail(WS_ERR_ALLOC, "cudaMallocHost failed");
   }
   return WS_OK;
 }
@@ -930,7 +973,7 @@ ws_status_t ws_csr_destroy(ws_csr_t h) {
     h->plan->ew.release();
     h->plan->sv.release();
     h->plan->rcd.release();
-    if (h->plan->host_sum) cudaFreeHost(h->plan->host_sum);
+    release_host_sum(h->plan->host_sum);
     delete h->plan;
   }
   delete h;
