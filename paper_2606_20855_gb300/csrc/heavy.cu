@@ -200,11 +200,216 @@ __device__ __forceinline__ long long first_at_least(const int32_t* cols, long lo
   return lo;
 }
 
+// Compact window for a dense heavy row whose output fits a few value windows
+// (nnz(row) <= kCompactPasses * width): the window is indexed by output
+// position instead of column, so the row needs no column slices; a row with
+// more entries than one window takes one pass of step 4-5 per window of
+// positions.  The flag bytes serve as a bitmap over the row's range
+// (8 * width bits >= 65,536 columns).
+//   1. warp 0 lists the stored A entries and cuts their whole B rows into
+//      pieces of kRcdPiece entries (scan of the piece counts into e_pp);
+//   2. the warps share the pieces and set the bit of every product column;
+//   3. each thread ranks a run of bitmap words (one barrier for the CTA
+//      scan), keeps the rank of every word (uint16) and writes the row's
+//      column indices in order;
+//   4. the warps take the pieces again and add a * b at the rank of each
+//      column (shared-memory atomics);
+//   5. the window is copied to C's values with coalesced stores and cleared;
+//      after the last pass every thread clears its bitmap words.
+// All threads of the CTA call it; the caller's barrier follows.  Returns
+// false, having written only the entry cache, when the extra walks of a
+// multi-pass row would cost more than column slices.
+constexpr int kRcdPiece = 128;  // B entries of one warp-sized piece
+constexpr int kCompactPre = 6400;  // byte offset of the word ranks in the entry cache
+constexpr int kCompactPasses = 2;  // value windows a compact row may take
+constexpr long long kCompactExtraProducts = 65536;  // products re-walked by the extra passes, at most
+
 template <typename T>
-__global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const RowPlan<T> p, int width) {
+__device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, unsigned char* cache, int width,
+                                int64_t ra, int na, long long lo, long long hi, int64_t cbase, int64_t cend,
+                                long long* s_cnt, int* s_work, bool* bad) {
+  constexpr int kWarps = kRcdNumThreads / 32;
+  constexpr int kPerLane = kRcdMegaA / 32;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  long long* e_b0 = reinterpret_cast<long long*>(cache);              // kRcdMegaA B row starts
+  T* e_av = reinterpret_cast<T*>(cache + kRcdMegaA * 8);              // kRcdMegaA A values
+  int* e_pp = reinterpret_cast<int*>(cache + kRcdMegaA * 16);         // first piece of every entry
+  int* e_len = e_pp + kRcdMegaA + 1;                                  // B row lengths
+  uint16_t* pre = reinterpret_cast<uint16_t*>(cache + kCompactPre);  // rank of every bitmap word
+  uint32_t* bm = reinterpret_cast<uint32_t*>(flags);
+  const int nnz = static_cast<int>(cend - cbase);
+  // 1. entries and pieces
+  if (warp == 0) {
+    int np[kPerLane];
+    int run = 0;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int j = lane * kPerLane + u;
+      np[u] = 0;
+      if (j < na) {
+        const int k = p.A.colidx[ra + j];
+        const long long b0 = p.B.rowptr[k];
+        const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        e_b0[j] = b0;
+        e_av[j] = p.A.vals[ra + j];
+        e_len[j] = len;
+        np[u] = (len + kRcdPiece - 1) / kRcdPiece;
+      }
+      run += np[u];
+    }
+    int incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    int at = incl - run;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int j = lane * kPerLane + u;
+      if (j < na) e_pp[j] = at;
+      at += np[u];
+    }
+    if (lane == 31) s_work[0] = incl;
+    long long prod = 0;  // the row's products
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int j = lane * kPerLane + u;
+      if (j < na) prod += e_len[j];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) prod += __shfl_xor_sync(kFull, prod, o);
+    if (lane == 0) s_work[1] = static_cast<int>(min(prod, static_cast<long long>(INT_MAX)));
+  }
+  __syncthreads();
+  const int npieces = s_work[0];
+  // Every window pass after the first walks all products again; past the
+  // budget the column-sliced path (one walk) is cheaper.
+  const int passes = (nnz + width - 1) / width;
+  if (static_cast<long long>(passes - 1) * s_work[1] > kCompactExtraProducts) return false;
+  // 2. bitmap of the product columns
+  for (int pc = warp; pc < npieces; pc += kWarps) {
+    int jl = 0, jh = na - 1;  // the entry of the piece: last one whose first piece is <= pc
+    while (jl < jh) {         // O(log na) probes of shared memory
+      const int mid = (jl + jh + 1) >> 1;
+      if (e_pp[mid] <= pc) {
+        jl = mid;
+      } else {
+        jh = mid - 1;
+      }
+    }
+    const int t0 = (pc - e_pp[jl]) * kRcdPiece + lane;
+    const int e = min((pc - e_pp[jl] + 1) * kRcdPiece, e_len[jl]);
+    const long long b = e_b0[jl];
+    int cc[kRcdPiece / 32];
+#pragma unroll
+    for (int u = 0; u < kRcdPiece / 32; ++u) cc[u] = t0 + u * 32 < e ? p.B.colidx[b + t0 + u * 32] : -1;
+#pragma unroll
+    for (int u = 0; u < kRcdPiece / 32; ++u) {
+      const long long off = cc[u] - lo;
+      if (cc[u] >= 0) {
+        if (off >= 0 && off <= hi - lo) {
+          atomicOr(bm + (off >> 5), 1u << (off & 31));
+        } else {
+          *bad = true;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  // 3. word ranks and C's column indices; thread t owns the bitmap words
+  // [4 t, 4 t + 4) (the range has at most 4 * kRcdNumThreads words; words
+  // past it are zero)
+  const int w0 = threadIdx.x * 4;
+  const uint4 v4 = *reinterpret_cast<const uint4*>(bm + w0);
+  const uint32_t wv[4] = {v4.x, v4.y, v4.z, v4.w};
+  const int mine = __popc(wv[0]) + __popc(wv[1]) + __popc(wv[2]) + __popc(wv[3]);
+  int incl = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) s_cnt[warp] = incl;
+  __syncthreads();
+  int run = incl - mine, total = 0;
+#pragma unroll
+  for (int v = 0; v < kWarps; ++v) {
+    const int n = static_cast<int>(s_cnt[v]);
+    run += v < warp ? n : 0;
+    total += n;
+  }
+  if (total != nnz) *bad = true;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int w = w0 + q;
+    pre[w] = static_cast<uint16_t>(run);
+    for (uint32_t m = wv[q]; m; m &= m - 1u) {
+      if (run < nnz) p.c_colidx[cbase + run] = static_cast<int32_t>(lo + (static_cast<long long>(w) << 5) + __ffs(m) - 1);
+      ++run;
+    }
+  }
+  __syncthreads();
+  // 4. values at the ranks of their columns, one window of ranks per pass
+  for (int q0 = 0; q0 < nnz; q0 += width) {
+    for (int pc = warp; pc < npieces; pc += kWarps) {
+      int jl = 0, jh = na - 1;
+      while (jl < jh) {  // O(log na) probes of shared memory
+        const int mid = (jl + jh + 1) >> 1;
+        if (e_pp[mid] <= pc) {
+          jl = mid;
+        } else {
+          jh = mid - 1;
+        }
+      }
+      const int t0 = (pc - e_pp[jl]) * kRcdPiece + lane;
+      const int e = min((pc - e_pp[jl] + 1) * kRcdPiece, e_len[jl]);
+      const long long b = e_b0[jl];
+      const T av = e_av[jl];
+      int cc[kRcdPiece / 32];
+      T bv[kRcdPiece / 32];
+#pragma unroll
+      for (int u = 0; u < kRcdPiece / 32; ++u) {
+        const int t = t0 + u * 32;
+        cc[u] = t < e ? p.B.colidx[b + t] : -1;
+        bv[u] = t < e ? p.B.vals[b + t] : T(0);
+      }
+#pragma unroll
+      for (int u = 0; u < kRcdPiece / 32; ++u) {
+        const long long off = cc[u] - lo;
+        if (cc[u] >= 0 && off >= 0 && off <= hi - lo) {
+          const int w = static_cast<int>(off >> 5);
+          const int rank = pre[w] + __popc(bm[w] & ((1u << (off & 31)) - 1u)) - q0;
+          if (rank >= 0 && rank < width) atomicAdd(dense + rank, av * bv[u]);
+        }
+      }
+    }
+    __syncthreads();
+    // 5. copy the window out and clear it
+    const int n = min(width, nnz - q0);
+    for (int i = threadIdx.x; i < n; i += kRcdNumThreads) {
+      p.c_vals[cbase + q0 + i] = dense[i];
+      dense[i] = T(0);
+    }
+    __syncthreads();
+  }
+  *reinterpret_cast<uint4*>(bm + w0) = make_uint4(0u, 0u, 0u, 0u);
+  return true;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kRcdNumThreads, 2) rcd_numeric_kernel(const RowPlan<T> p, int width) {
   constexpr int kS = rcd_slices<T>();
   static_assert(kRcdCacheA * (2 * sizeof(long long) + sizeof(T) + sizeof(int)) <= kRcdMaxA * sizeof(int),
                 "the entry cache fits the space after the window");
+  static_assert(kRcdMegaA * 16 + (2 * kRcdMegaA + 1) * static_cast<int>(sizeof(int)) <= kCompactPre &&
+                    kCompactPre + kMaxBitmapSpan / 32 * sizeof(uint16_t) <=
+                        kRcdCacheA * (2 * sizeof(long long) + sizeof(T) + sizeof(int)),
+                "the compact-window layout fits the entry cache");
+  static_assert(kMaxBitmapSpan <= 65536, "a row has at most 65,536 entries, so word ranks fit uint16");
+  static_assert(kRcdWidthBytes / static_cast<int>(sizeof(T)) * 8 >= kMaxBitmapSpan &&
+                    kMaxBitmapSpan / 32 == 4 * kRcdNumThreads,
+                "the flag bytes hold a bitmap of the range; four bitmap words per thread");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   T* dense = reinterpret_cast<T*>(smem_raw);                           // width values
   uint8_t* flags = smem_raw + static_cast<size_t>(width) * sizeof(T);  // width bytes
@@ -213,7 +418,7 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
   T* c_av = reinterpret_cast<T*>(c_end + kRcdCacheA);                  //   the A value,
   int* c_long = reinterpret_cast<int*>(c_av + kRcdCacheA);             //   and the list of long parts
   __shared__ long long s_scan[32];
-  __shared__ int s_item, s_next, s_next2, s_nlong;
+  __shared__ int s_item, s_next, s_next2, s_nlong, s_work[2];
   __shared__ long long s_out0;
   const int lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < width; i += kRcdNumThreads) {
@@ -315,6 +520,10 @@ __global__ void __launch_bounds__(kRcdNumThreads, 1) rcd_numeric_kernel(const Ro
     const long long lo = p.lo[row], hi = p.hi[row];
     const int64_t cbase = p.c_rowptr[row];
     const int64_t cend = p.c_rowptr[row + 1];
+    if (cend - cbase <= static_cast<int64_t>(kCompactPasses) * width &&
+        rcd_compact_row(p, dense, flags, reinterpret_cast<unsigned char*>(c_pos), width, ra, na, lo, hi, cbase, cend,
+                        s_scan, s_work, &bad))
+      continue;  // done without column slices
     for (int j = threadIdx.x; j < na; j += kRcdNumThreads) {
       const int k = p.A.colidx[ra + j];
       c_pos[j] = p.B.rowptr[k];

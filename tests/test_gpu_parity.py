@@ -150,6 +150,50 @@ def test_heavy_rows(heavy, dtype):
 
 
 @pytest.mark.parametrize("dtype", DTYPES)
+def test_dense_rows_slice_parts(dtype):
+    """Dense heavy rows whose B rows give every kind of part inside a value
+    window slice: empty, one entry, just below / at / just above the short-part
+    limit (32) and the piece size (128), many pieces, a B row covering all
+    65,536 columns, columns on the slice starts and just before them, a B row
+    inside one slice; one row with more than 256 stored entries; and rows
+    whose output is below, exactly at and one above the value window's size
+    (the compact window takes the first two)."""
+    rng = np.random.default_rng(33)
+    n = 1 << 16
+    slice_w = 8192 if dtype == np.float64 else 16384
+    lens = [0, 1, 2, 31, 32, 33, 127, 128, 129, 257, 1000, 4000, 20000]
+    rows = {i: rng.choice(n, size=L, replace=False).tolist() for i, L in enumerate(lens)}
+    rows[len(lens)] = list(range(n))                                       # every column
+    rows[len(lens) + 1] = [s * slice_w + d for s in range(n // slice_w) for d in (-1, 0) if 0 <= s * slice_w + d < n]
+    rows[len(lens) + 2] = (3 * slice_w + rng.choice(slice_w, size=300, replace=False)).tolist()  # one slice
+    x = rng.permutation(n)[:slice_w]                      # exactly one window of distinct columns
+    rows[len(lens) + 3] = x.tolist()
+    rows[len(lens) + 4] = rng.choice(x, size=500, replace=False).tolist()            # inside x
+    outside = np.setdiff1d(np.arange(n), x)
+    rows[len(lens) + 5] = rng.choice(x, size=100, replace=False).tolist() + [int(outside[7])]  # one column more
+    k = 400
+    for i in range(len(lens) + 6, k):
+        rows[i] = rng.choice(n, size=int(rng.integers(0, 300)), replace=False).tolist()
+    B = _csr(k, n, rows, dtype=dtype)
+    B.vals = (2 * rng.random(B.nnz) - 1).astype(dtype)
+    special = list(range(len(lens) + 3))
+    X = len(lens) + 3
+    arows = {0: special, 1: special[:5] + [len(lens)], 2: [len(lens) + 1, len(lens) + 2, 12],
+             3: rng.choice(k, size=300, replace=False).tolist(),                 # 300 > 256 entries
+             4: [6, 7, 8, 9, 10, 11],                 # output fits one value window
+             5: [X, X + 1],                           # output exactly one window wide
+             6: [X, X + 2]}                           # one column more than a window
+    for i in range(7, 40):
+        arows[i] = rng.choice(k, size=int(rng.integers(2, 200)), replace=False).tolist() + [12]
+    A = _csr(40, k, arows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["rcd_rows"] >= 38
+    assert np.diff(rowptr)[5] == slice_w and np.diff(rowptr)[6] == slice_w + 1
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
 def test_wide_heavy_rows(dtype):
     """Rows with thousands of stored A entries over short B rows spanning ~2^20 columns."""
     rng = np.random.default_rng(32)
