@@ -144,6 +144,7 @@ struct Plan {
   DevBuf ew;      // elementwise operations: summary, chunk arrays, scan partials
   DevBuf sv;      // sparse matrix - sparse vector product (in A^T's handle): accumulator, byte-map, offsets
   DevBuf rcd;     // dense heavy rows: per-slice counts, mega-row list, work counters
+  DevBuf rcdb;    // dense heavy rows: slice starts of the mega rows' B rows
   int kind = kPlanNone;  // which symbolic pass filled this plan
   // elementwise plan (kPlanEwise)
   int ew_op = 0, ew_group = 32;
@@ -156,6 +157,9 @@ struct Plan {
   int32_t* rcd_mega = nullptr;
   int32_t* rcd_nmega = nullptr;
   int32_t* rcd_ctr = nullptr;
+  int64_t* rcd_moff = nullptr;
+  int32_t* rcd_mna = nullptr;
+  long long rcd_mega_entries = 0;
   // submatrix plan (kPlanSub): the block the symbolic pass counted
   int64_t sub_r0 = 0, sub_r1 = 0, sub_c0 = 0, sub_c1 = 0;
   DevSummary* host_sum = nullptr;  // pinned
@@ -332,17 +336,23 @@ ws_status_t symbolic_bins(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
     const int64_t nr = pl->seg_count[kSegRcd];
     const size_t o_scnt = 0;
     const size_t o_mega = align_up(o_scnt + 4 * static_cast<size_t>(nr) * rcd_slices<T>(), 256);
-    const size_t o_cnt = align_up(o_mega + 4 * static_cast<size_t>(nr), 256);
+    const size_t o_moff = align_up(o_mega + 4 * static_cast<size_t>(nr), 256);
+    const size_t o_mna = align_up(o_moff + 8 * static_cast<size_t>(nr), 256);
+    const size_t o_cnt = align_up(o_mna + 4 * static_cast<size_t>(nr), 256);
     st = pl->rcd.reserve(o_cnt + 256, s);
     if (st != WS_OK) return st;
     char* b = static_cast<char*>(pl->rcd.ptr);
     pl->rcd_scnt = reinterpret_cast<int32_t*>(b + o_scnt);
     pl->rcd_mega = reinterpret_cast<int32_t*>(b + o_mega);
+    pl->rcd_moff = reinterpret_cast<int64_t*>(b + o_moff);
+    pl->rcd_mna = reinterpret_cast<int32_t*>(b + o_mna);
     pl->rcd_nmega = reinterpret_cast<int32_t*>(b + o_cnt);
     pl->rcd_ctr = pl->rcd_nmega + 1;
     WS_CUDA(cudaMemsetAsync(pl->rcd_nmega, 0, sizeof(int32_t), s), "cudaMemsetAsync(rcd counters)");
     p.rcd_scnt = pl->rcd_scnt;
     p.rcd_mega = pl->rcd_mega;
+    p.rcd_moff = pl->rcd_moff;
+    p.rcd_mna = pl->rcd_mna;
     p.rcd_nmega = pl->rcd_nmega;
     p.rcd_ctr = pl->rcd_ctr;
     p.seg_begin = pl->seg_offset[kSegRcd];
@@ -446,6 +456,7 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
   st = device_status(*pl->host_sum);
   if (st != WS_OK) return st;
   pl->n_sort = pl->host_sum->n_sort;
+  pl->rcd_mega_entries = pl->all_planned ? 0 : pl->host_sum->rcd_mega_entries;
   C->nnz = m > 0 ? pl->host_sum->nnz : 0;
   pl->A = A;
   pl->B = B;
@@ -477,10 +488,19 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     WS_CUDA(cudaMemsetAsync(pl->rcd_ctr, 0, 2 * sizeof(int32_t), s), "cudaMemsetAsync(rcd work counters)");
     p.rcd_scnt = pl->rcd_scnt;
     p.rcd_mega = pl->rcd_mega;
+    p.rcd_moff = pl->rcd_moff;
+    p.rcd_mna = pl->rcd_mna;
     p.rcd_nmega = pl->rcd_nmega;
     p.rcd_ctr = pl->rcd_ctr;
     p.seg_begin = pl->seg_offset[kSegRcd];
     p.seg_len = pl->seg_count[kSegRcd];
+    if (pl->rcd_mega_entries > 0) {  // slice starts of the mega rows' B rows, found once per entry
+      const size_t need = static_cast<size_t>(pl->rcd_mega_entries) * (rcd_slices<T>() - 1) * sizeof(int32_t);
+      ws_status_t st = pl->rcdb.reserve(need > 0 ? need : 4, s);
+      if (st != WS_OK) return st;
+      p.rcd_bnd = static_cast<int32_t*>(pl->rcdb.ptr);
+      launch_rcd_bounds<T>(p, sms, s, &pl->num_launches);
+    }
     launch_rcd<T>(p, true, sms, s, &pl->num_launches);
   }
   if (pl->seg_count[kSegWb] > 0) {
@@ -965,7 +985,7 @@ ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
     if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr || h->plan->sv.ptr ||
-        h->plan->rcd.ptr)
+        h->plan->rcd.ptr || h->plan->rcdb.ptr)
       cudaDeviceSynchronize();
     h->plan->rows.release();
     h->plan->slices.release();
@@ -973,6 +993,7 @@ ws_status_t ws_csr_destroy(ws_csr_t h) {
     h->plan->ew.release();
     h->plan->sv.release();
     h->plan->rcd.release();
+    h->plan->rcdb.release();
     release_host_sum(h->plan->host_sum);
     delete h->plan;
   }

@@ -97,7 +97,13 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
     block_exclusive_scan(cnt, s_scan, &total);
     if (threadIdx.x == 0) {
       p.c_rowptr[row + 1] = total;
-      if (re - ra > kRcdMegaA) p.rcd_mega[atomicAdd(p.rcd_nmega, 1)] = static_cast<int32_t>(r);
+      if (re - ra > kRcdMegaA) {
+        const int idx = atomicAdd(p.rcd_nmega, 1);
+        p.rcd_mega[idx] = static_cast<int32_t>(r);
+        p.rcd_mna[idx] = static_cast<int32_t>(re - ra);
+        p.rcd_moff[idx] = static_cast<int64_t>(
+            atomicAdd(reinterpret_cast<unsigned long long*>(&p.sum->rcd_mega_entries), static_cast<unsigned long long>(re - ra)));
+      }
     }
     if (threadIdx.x < kS) {
       p.rcd_scnt[r * kS + threadIdx.x] = s_slice[threadIdx.x];
@@ -107,19 +113,85 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
   }
 }
 
+// Slice starts of the mega rows' B rows, found once per stored A entry
+// instead of once per (row, slice) item.  Block b takes mega rows b,
+// b + gridDim.x, ...; thread j the row's entries j, j + blockDim.x, ...: for
+// every slice start lo + s * width (s = 1 .. ns - 1) the first position of the
+// sorted B row at or past it, the ns - 1 binary searches run in lockstep so
+// their loads are in flight together.  Row idx's table holds (kS - 1) arrays
+// of its na entries, slice by slice, from rcd_moff[idx] * (kS - 1).
+template <typename T>
+__global__ void __launch_bounds__(kRcdNumThreads) rcd_bounds_kernel(const RowPlan<T> p, int width) {
+  constexpr int kS = rcd_slices<T>();
+  const int n_mega = *p.rcd_nmega;
+  for (int idx = blockIdx.x; idx < n_mega; idx += gridDim.x) {
+    const int32_t row = p.perm[p.seg_begin + p.rcd_mega[idx]];
+    const long long lo = p.lo[row], hi = p.hi[row];
+    const int ns = static_cast<int>((hi - lo + width) / width);
+    const int64_t ra = p.A.rowptr[row];
+    const int na = p.rcd_mna[idx];
+    if (p.A.rowptr[row + 1] - ra != na) continue;  // the input changed: the numeric item reports it
+    int32_t* tab = p.rcd_bnd + p.rcd_moff[idx] * (kS - 1);
+    for (int j = threadIdx.x; j < na; j += blockDim.x) {
+      const int k = p.A.colidx[ra + j];
+      const int64_t b0 = p.B.rowptr[k];
+      const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+      const int32_t* cols = p.B.colidx + b0;
+      int slo[kS], shi[kS];
+#pragma unroll
+      for (int q = 1; q < kS; ++q) {
+        slo[q] = 0;
+        shi[q] = q < ns ? len : 0;
+      }
+      for (int round = 0; round < 64; ++round) {  // each search halves its interval: <= 32 rounds
+        int v[kS];
+        bool open = false;
+#pragma unroll
+        for (int q = 1; q < kS; ++q) {
+          v[q] = 0;
+          if (slo[q] < shi[q]) {
+            open = true;
+            v[q] = cols[(slo[q] + shi[q]) >> 1];
+          }
+        }
+        if (!open) break;
+#pragma unroll
+        for (int q = 1; q < kS; ++q) {
+          if (slo[q] < shi[q]) {
+            const int mid = (slo[q] + shi[q]) >> 1;
+            if (v[q] < lo + static_cast<long long>(q) * width) {
+              slo[q] = mid + 1;
+            } else {
+              shi[q] = mid;
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 1; q < kS; ++q) {
+        if (q < ns) tab[static_cast<int64_t>(q - 1) * na + j] = slo[q];
+      }
+    }
+  }
+}
+
 // Numeric pass of the dense heavy rows.  Two kinds of work, taken from two
 // counters so CTAs balance themselves:
 //   1. mega rows (more than kRcdMegaA stored A entries, typically the hub
 //      rows of a power-law matrix): every (row, slice) pair is a separate
-//      item, so one row's slices run on several CTAs at once.  An item finds
-//      the part of each entry's B row inside its slice by binary search
-//      (one lane per entry, kRcdBatch entries at a time), walks the long
-//      parts with a warp each and the short ones with a lane each, and emits
-//      the slice from the offset the symbolic pass's per-slice counts give.
-//   2. the other rows: one CTA per row, slices in order; each entry's B-row
-//      position, end and A value stay in shared memory for the whole row and
-//      every slice continues where the last one stopped.
-constexpr int kRcdShort = 32;  // parts of B rows walked by a single lane
+//      item, so one row's slices run on several CTAs at once.  An item reads
+//      the part of each entry's B row inside its slice from the table of
+//      slice starts (rcd_bounds_kernel), walks the long parts with a warp
+//      each and the short ones with a group of lanes each, and emits the
+//      slice from the offset the symbolic pass's per-slice counts give.
+//   2. the other rows, one CTA per row.  A row whose output fits one or two
+//      value windows takes the compact window (rcd_compact_row: no column
+//      slices); the others go slice by slice, each entry's B-row position,
+//      end and A value staying in shared memory for the whole row and every
+//      slice continuing where the last one stopped.
+constexpr int kRcdShort = 32;  // parts of B rows walked by one group of kShortLanes lanes
+constexpr int kShortLanes = 8;  // lanes walking one short part, four entries each
+static_assert(kShortLanes * 4 >= kRcdShort, "a short part takes one round of loads");
 
 // Emits one slice of the dense window in column order: thread t owns the
 // contiguous 16-byte flag chunks [t * cpt, (t + 1) * cpt); it counts their set
@@ -186,20 +258,6 @@ __device__ __forceinline__ void rcd_warp_add(const RowPlan<T>& p, T* dense, uint
   }
 }
 
-// First position in cols[0..n) with cols[pos] >= c (n if none).
-__device__ __forceinline__ long long first_at_least(const int32_t* cols, long long n, long long c) {
-  long long lo = 0, hi = n;
-  while (lo < hi) {  // O(log n) probes
-    const long long mid = (lo + hi) >> 1;
-    if (cols[mid] < c) {
-      lo = mid + 1;
-    } else {
-      hi = mid;
-    }
-  }
-  return lo;
-}
-
 // Compact window for a dense heavy row whose output fits a few value windows
 // (nnz(row) <= kCompactPasses * width): the window is indexed by output
 // position instead of column, so the row needs no column slices; a row with
@@ -209,9 +267,10 @@ __device__ __forceinline__ long long first_at_least(const int32_t* cols, long lo
 //   1. warp 0 lists the stored A entries and cuts their whole B rows into
 //      pieces of kRcdPiece entries (scan of the piece counts into e_pp);
 //   2. the warps share the pieces and set the bit of every product column;
-//   3. each thread ranks a run of bitmap words (one barrier for the CTA
-//      scan), keeps the rank of every word (uint16) and writes the row's
-//      column indices in order;
+//   3. each thread ranks four consecutive bitmap words (one barrier for
+//      the CTA scan) and keeps the rank of every word (uint16); after a
+//      barrier each thread writes the column indices of four words strided
+//      by the CTA size (a dense stretch of columns is shared out);
 //   4. the warps take the pieces again and add a * b at the rank of each
 //      column (shared-memory atomics);
 //   5. the window is copied to C's values with coalesced stores and cleared;
@@ -219,7 +278,7 @@ __device__ __forceinline__ long long first_at_least(const int32_t* cols, long lo
 // All threads of the CTA call it; the caller's barrier follows.  Returns
 // false, having written only the entry cache, when the extra walks of a
 // multi-pass row would cost more than column slices.
-constexpr int kRcdPiece = 128;  // B entries of one warp-sized piece
+constexpr int kRcdPiece = 256;  // B entries of one warp-sized piece
 constexpr int kCompactPre = 6400;  // byte offset of the word ranks in the entry cache
 constexpr int kCompactPasses = 2;  // value windows a compact row may take
 constexpr long long kCompactExtraProducts = 65536;  // products re-walked by the extra passes, at most
@@ -342,14 +401,22 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
   if (total != nnz) *bad = true;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    const int w = w0 + q;
-    pre[w] = static_cast<uint16_t>(run);
-    for (uint32_t m = wv[q]; m; m &= m - 1u) {
-      if (run < nnz) p.c_colidx[cbase + run] = static_cast<int32_t>(lo + (static_cast<long long>(w) << 5) + __ffs(m) - 1);
-      ++run;
-    }
+    pre[w0 + q] = static_cast<uint16_t>(run);
+    run += __popc(wv[q]);
   }
   __syncthreads();
+  // Column indices in order: thread t writes those of the words t, t + 512,
+  // t + 1024, t + 1536 (strided, so a dense stretch of columns is shared out).
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int w = q * kRcdNumThreads + threadIdx.x;
+    const long long col0 = lo + (static_cast<long long>(w) << 5) - 1;
+    int at = pre[w];
+    for (uint32_t m = bm[w]; m; m &= m - 1u) {
+      if (at < nnz) p.c_colidx[cbase + at] = static_cast<int32_t>(col0 + __ffs(m));
+      ++at;
+    }
+  }
   // 4. values at the ranks of their columns, one window of ranks per pass
   for (int q0 = 0; q0 < nnz; q0 += width) {
     for (int pc = warp; pc < npieces; pc += kWarps) {
@@ -451,16 +518,25 @@ __global__ void __launch_bounds__(kRcdNumThreads, 2) rcd_numeric_kernel(const Ro
     }
     const int64_t ra = p.A.rowptr[row];
     const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
+    const int ns = static_cast<int>((hi - lo + width) / width);
+    const int32_t* tab = p.rcd_bnd + p.rcd_moff[item / kS] * (kS - 1);
+    if (na != p.rcd_mna[item / kS]) {  // the input changed since the symbolic pass
+      bad = true;
+      continue;
+    }
     for (int e0 = 0; e0 < na; e0 += kRcdCacheA) {
       const int nb = min(kRcdCacheA, na - e0);
+      // the part of each entry's B row inside the slice, from the table of
+      // slice starts (rcd_bounds_kernel)
       for (int j = threadIdx.x; j < nb; j += kRcdNumThreads) {
-        const int k = p.A.colidx[ra + e0 + j];
+        const int e = e0 + j;
+        const int k = p.A.colidx[ra + e];
         const long long b0 = p.B.rowptr[k], len = p.B.rowptr[k + 1] - b0;
-        const long long st = first_at_least(p.B.colidx + b0, len, c0);
-        const long long en = st + first_at_least(p.B.colidx + b0 + st, len - st, c1);
+        const long long st = sl == 0 ? 0 : tab[static_cast<int64_t>(sl - 1) * na + e];
+        const long long en = sl + 1 < ns ? tab[static_cast<int64_t>(sl) * na + e] : len;
         c_pos[j] = b0 + st;
         c_end[j] = b0 + en;
-        c_av[j] = p.A.vals[ra + e0 + j];
+        c_av[j] = p.A.vals[ra + e];
         if (en - st > kRcdShort) c_long[atomicAdd(&s_nlong, 1)] = j;
       }
       if (threadIdx.x == 0) {
@@ -477,18 +553,33 @@ __global__ void __launch_bounds__(kRcdNumThreads, 2) rcd_numeric_kernel(const Ro
         const int j = c_long[t];
         rcd_warp_add(p, dense, flags, c_pos[j], c_end[j] - c_pos[j], c_av[j], c0, lane);
       }
-      for (int g2 = 0; g2 <= nb / 32 + 1; ++g2) {  // short parts: a lane each
+      // short parts: a group of kShortLanes lanes each, every lane loading up
+      // to four of the part's entries at once (one round of loads per part)
+      constexpr int kGroupsPerWarp = 32 / kShortLanes;
+      for (int g2 = 0; g2 <= nb / kGroupsPerWarp + 1; ++g2) {
         int base = 0;
-        if (lane == 0) base = atomicAdd(&s_next2, 32);
+        if (lane == 0) base = atomicAdd(&s_next2, kGroupsPerWarp);
         base = __shfl_sync(kFull, base, 0);
         if (base >= nb) break;
-        const int j = base + lane;
+        const int j = base + lane / kShortLanes;
         if (j < nb && c_end[j] - c_pos[j] <= kRcdShort) {
           const T av = c_av[j];
-          for (long long t = c_pos[j]; t < c_end[j]; ++t) {
-            const int off = static_cast<int>(p.B.colidx[t] - c0);
-            atomicAdd(dense + off, av * p.B.vals[t]);
-            flags[off] = 1;
+          const long long t0 = c_pos[j] + lane % kShortLanes, e = c_end[j];
+          int cc[4];
+          T bv[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const long long t = t0 + u * kShortLanes;
+            cc[u] = t < e ? p.B.colidx[t] : -1;
+            bv[u] = t < e ? p.B.vals[t] : T(0);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (cc[u] >= 0) {
+              const int off = static_cast<int>(cc[u] - c0);
+              atomicAdd(dense + off, av * bv[u]);
+              flags[off] = 1;
+            }
           }
         }
       }
@@ -764,6 +855,13 @@ void launch_rcd(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, 
 }
 
 template <typename T>
+void launch_rcd_bounds(const RowPlan<T>& p, int num_sms, cudaStream_t s, int* launches) {
+  const int width = kRcdWidthBytes / static_cast<int>(sizeof(T));
+  rcd_bounds_kernel<T><<<grid_of(p.seg_len, num_sms, 4), kRcdNumThreads, 0, s>>>(p, width);
+  *launches += 1;
+}
+
+template <typename T>
 void launch_wb(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches) {
   const size_t smem = kWbMaxSpan / 8 + (kWbMaxSpan / 128) * 4;
   auto kern = numeric ? wb_kernel<T, true> : wb_kernel<T, false>;
@@ -775,6 +873,8 @@ void launch_wb(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, i
 
 template void launch_rcd<float>(const RowPlan<float>&, bool, int, cudaStream_t, int*);
 template void launch_rcd<double>(const RowPlan<double>&, bool, int, cudaStream_t, int*);
+template void launch_rcd_bounds<float>(const RowPlan<float>&, int, cudaStream_t, int*);
+template void launch_rcd_bounds<double>(const RowPlan<double>&, int, cudaStream_t, int*);
 template void launch_wb<float>(const RowPlan<float>&, bool, int, cudaStream_t, int*);
 template void launch_wb<double>(const RowPlan<double>&, bool, int, cudaStream_t, int*);
 

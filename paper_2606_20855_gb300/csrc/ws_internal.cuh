@@ -109,6 +109,7 @@ struct DevSummary {
   long long products;  // sum of ub_i
   long long dense_slices;
   long long slice_cursor;
+  long long rcd_mega_entries;  // stored A entries of the dense heavy rows split into (row, slice) items
   int status;
   int n_sort;
   int n_long;
@@ -146,9 +147,12 @@ struct RowPlan {
   int32_t* slice_cnt;          // entries per dense-window slice
   uint16_t* ranks;             // register bitmap rows: output position of every product, kBmrSlots per row
   int32_t* rcd_scnt;           // dense heavy rows: entries per dense-window slice, rcd_slices<T>() per row
-  int32_t* rcd_mega;           // dense heavy rows with more than 1024 stored A entries (segment positions)
+  int32_t* rcd_mega;           // dense heavy rows with more than 256 stored A entries (segment positions)
   int32_t* rcd_nmega;          // their number
   int32_t* rcd_ctr;            // two work counters of the numeric kernel (zeroed before it)
+  int64_t* rcd_moff;           // per mega row: first of its entries in the slice-start table
+  int32_t* rcd_mna;            // per mega row: its stored A entries when the table was sized
+  int32_t* rcd_bnd;            // slice-start table of the mega rows' B rows (numeric only)
   DevSummary* sum;
   int64_t seg_begin;   // first position in perm of the segment a kernel processes
   int64_t seg_len;     // rows in that segment
@@ -250,6 +254,8 @@ template <typename T>
 void launch_bitmap(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_rcd(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches);
+template <typename T>
+void launch_rcd_bounds(const RowPlan<T>& p, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
 void launch_wb(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, int* launches);
 template <typename T>
