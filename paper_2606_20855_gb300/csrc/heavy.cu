@@ -70,18 +70,44 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
     const int lo = p.lo[row];
     const int span = p.hi[row] - lo + 1;
     const int64_t ra = p.A.rowptr[row], re = p.A.rowptr[row + 1];
-    for (int64_t pa = ra + warp; pa < re; pa += kWarps) {
-      const int k = p.A.colidx[pa];
-      const int64_t qe = p.B.rowptr[k + 1];
-      int64_t q = p.B.rowptr[k] + lane;
-      for (; q + 96 < qe; q += 128) {  // four loads in flight per lane
-        const int c0 = p.B.colidx[q], c1 = p.B.colidx[q + 32], c2 = p.B.colidx[q + 64], c3 = p.B.colidx[q + 96];
-        flags[c0 - lo] = 1;
-        flags[c1 - lo] = 1;
-        flags[c2 - lo] = 1;
-        flags[c3 - lo] = 1;
+    // A warp takes four stored A entries per round, one per group of 8
+    // lanes: a B row of at most 32 entries is flagged by its group in one
+    // round of loads (four per lane), longer ones by the whole warp after.
+    for (int64_t pa0 = ra + static_cast<int64_t>(warp) * 4; pa0 < re; pa0 += kWarps * 4) {
+      const int64_t pa = pa0 + (lane >> 3);
+      int64_t qb = 0, qe = 0;
+      if (pa < re) {
+        const int k = p.A.colidx[pa];
+        qb = p.B.rowptr[k];
+        qe = p.B.rowptr[k + 1];
       }
-      for (; q < qe; q += 32) flags[p.B.colidx[q] - lo] = 1;
+      const bool lng = qe - qb > 32;
+      const unsigned longs = __ballot_sync(kFull, lng && (lane & 7) == 0);
+      if (!lng) {
+        int c[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t t = qb + (lane & 7) + 8 * u;
+          c[u] = t < qe ? p.B.colidx[t] : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          if (c[u] >= 0) flags[c[u] - lo] = 1;
+        }
+      }
+      for (unsigned m = longs; m; m &= m - 1u) {
+        const int src = __ffs(m) - 1;
+        const int64_t be = __shfl_sync(kFull, qe, src);
+        int64_t q = __shfl_sync(kFull, qb, src) + lane;
+        for (; q + 96 < be; q += 128) {  // four loads in flight per lane
+          const int c0 = p.B.colidx[q], c1 = p.B.colidx[q + 32], c2 = p.B.colidx[q + 64], c3 = p.B.colidx[q + 96];
+          flags[c0 - lo] = 1;
+          flags[c1 - lo] = 1;
+          flags[c2 - lo] = 1;
+          flags[c3 - lo] = 1;
+        }
+        for (; q < be; q += 32) flags[p.B.colidx[q] - lo] = 1;
+      }
     }
     __syncthreads();
     long long cnt = 0;
@@ -114,8 +140,10 @@ __global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowP
 }
 
 // Slice starts of the mega rows' B rows, found once per stored A entry
-// instead of once per (row, slice) item.  Block b takes mega rows b,
-// b + gridDim.x, ...; thread j the row's entries j, j + blockDim.x, ...: for
+// instead of once per (row, slice) item.  Blocks (b, y) take mega rows b,
+// b + gridDim.x, ...; thread t of block (b, y) the row's entries
+// y * blockDim.x + t, stepping by gridDim.y * blockDim.x (the gridDim.y blocks
+// of a row share its entries, so one long row is no tail): for
 // every slice start lo + s * width (s = 1 .. ns - 1) the first position of the
 // sorted B row at or past it, the ns - 1 binary searches run in lockstep so
 // their loads are in flight together.  Row idx's table holds (kS - 1) arrays
@@ -132,7 +160,7 @@ __global__ void __launch_bounds__(kRcdNumThreads) rcd_bounds_kernel(const RowPla
     const int na = p.rcd_mna[idx];
     if (p.A.rowptr[row + 1] - ra != na) continue;  // the input changed: the numeric item reports it
     int32_t* tab = p.rcd_bnd + p.rcd_moff[idx] * (kS - 1);
-    for (int j = threadIdx.x; j < na; j += blockDim.x) {
+    for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < na; j += gridDim.y * blockDim.x) {
       const int k = p.A.colidx[ra + j];
       const int64_t b0 = p.B.rowptr[k];
       const int len = static_cast<int>(p.B.rowptr[k + 1] - b0);
@@ -857,7 +885,9 @@ void launch_rcd(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s, 
 template <typename T>
 void launch_rcd_bounds(const RowPlan<T>& p, int num_sms, cudaStream_t s, int* launches) {
   const int width = kRcdWidthBytes / static_cast<int>(sizeof(T));
-  rcd_bounds_kernel<T><<<grid_of(p.seg_len, num_sms, 4), kRcdNumThreads, 0, s>>>(p, width);
+  constexpr int kBlocksPerRow = 8;
+  const dim3 grid(grid_of(p.seg_len, num_sms, 1), kBlocksPerRow);
+  rcd_bounds_kernel<T><<<grid, kRcdNumThreads, 0, s>>>(p, width);
   *launches += 1;
 }
 
