@@ -35,7 +35,7 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kRcdThreads = 256;
 constexpr int kRcdNumThreads = 512;
-constexpr int kWbThreads = 512;
+constexpr int kWbThreads = 1024;  // one CTA per SM (its 128 KB bitmap), so 32 warps hide the gathers
 constexpr int kWbBatch = 4;  // stored A entries a lane group has in flight in the wide-bitmap kernel
 
 // ---------------------------------------------------------------- dense rows
