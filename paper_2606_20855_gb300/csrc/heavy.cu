@@ -33,7 +33,7 @@ namespace wsk {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kRcdThreads = 256;
+constexpr int kRcdThreads = 512;
 constexpr int kRcdNumThreads = 512;
 constexpr int kWbThreads = 1024;  // one CTA per SM (its 128 KB bitmap), so 32 warps hide the gathers
 constexpr int kWbBatch = 4;  // stored A entries a lane group has in flight in the wide-bitmap kernel
@@ -53,7 +53,7 @@ __device__ __forceinline__ int nonzero_bytes(const uint4 v) {
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kRcdThreads, 2) rcd_symbolic_kernel(const RowPlan<T> p) {
+__global__ void __launch_bounds__(kRcdThreads, 3) rcd_symbolic_kernel(const RowPlan<T> p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint8_t* flags = smem_raw;  // kMaxBitmapSpan bytes
   uint4* flags4 = reinterpret_cast<uint4*>(smem_raw);
