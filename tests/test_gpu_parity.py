@@ -150,6 +150,29 @@ def test_heavy_rows(heavy, dtype):
 
 
 @pytest.mark.parametrize("dtype", DTYPES)
+def test_direct_rows_long_and_short(dtype):
+    """Rows of A with one stored entry copy a scaled B row: B rows of 0 to
+    5000 entries around the length where a whole warp takes over (512), among
+    many short ones so the lane groups stay small."""
+    rng = np.random.default_rng(34)
+    n = 20_000
+    lens = [0, 1, 3, 31, 32, 33, 511, 512, 513, 1000, 5000]
+    rows = {i: rng.choice(n, size=L, replace=False).tolist() for i, L in enumerate(lens)}
+    k = 3000
+    for i in range(len(lens), k):
+        rows[i] = rng.choice(n, size=int(rng.integers(1, 6)), replace=False).tolist()
+    B = _csr(k, n, rows, dtype=dtype)
+    B.vals = (2 * rng.random(B.nnz) - 1).astype(dtype)
+    picks = list(range(len(lens))) * 3 + rng.choice(k, size=400).tolist()
+    A = _csr(len(picks), k, {i: [c] for i, c in enumerate(picks)}, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    blen = np.diff(B.rowptr)
+    assert info["direct_rows"] == int(np.count_nonzero(blen[picks]))  # an empty B row gives an empty row
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
 def test_dense_rows_slice_parts(dtype):
     """Dense heavy rows whose B rows give every kind of part inside a value
     window slice: empty, one entry, just below / at / just above the short-part
