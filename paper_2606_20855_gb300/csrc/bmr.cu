@@ -241,9 +241,15 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const
 // of Sec. 4), and the warp copies the sorted row to C with coalesced stores.
 constexpr int kHdrRows = 8;
 
-template <typename T>
+// Staging slots of one warp: a row has at most kBmrMaxA * G products (the
+// lane groups of G lanes take kBmrMaxA stored A entries), so at most that
+// many entries; smaller groups need less shared memory and fit more warps.
+template <int G>
+constexpr int numeric_cap() { return kBmrMaxA * G; }
+
+template <typename T, int G>
 constexpr size_t numeric_warp_bytes() {
-  return static_cast<size_t>(kBmrCap) * (4 + sizeof(T)) +
+  return static_cast<size_t>(numeric_cap<G>()) * (4 + sizeof(T)) +
          static_cast<size_t>(kHdrRows) * kBmrMaxA * (sizeof(long long) + sizeof(int) + sizeof(T)) +
          static_cast<size_t>(kHdrRows) * (2 * sizeof(long long) + sizeof(int));
 }
@@ -258,10 +264,12 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int grp = lane / G, gl = lane % G;
-  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * numeric_warp_bytes<T>();
+  constexpr int kCap = numeric_cap<G>();
+  static_assert(kCap <= kBmrCap, "ranks fit the plan's 15 bits");
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * numeric_warp_bytes<T, G>();
   int* st_key = reinterpret_cast<int*>(ws);
-  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kBmrCap) * 4);
-  long long* h_b0 = reinterpret_cast<long long*>(ws + static_cast<size_t>(kBmrCap) * (4 + sizeof(T)));
+  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kCap) * 4);
+  long long* h_b0 = reinterpret_cast<long long*>(ws + static_cast<size_t>(kCap) * (4 + sizeof(T)));
   T* h_a = reinterpret_cast<T*>(h_b0 + kEnt);
   int* h_len = reinterpret_cast<int*>(h_a + kEnt);
   long long* h_cbase = reinterpret_cast<long long*>(h_len + kEnt);  // C offset and nnz of each batch row
@@ -309,8 +317,8 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
       if (row < 0) break;
       const long long cbase = h_cbase[i];
       const long long want = h_cnt[i];
-      const int cnt = static_cast<int>(want < kBmrCap ? want : kBmrCap);  // staging bounds every access
-      if (lane == 0 && want > kBmrCap) atomicOr(&p.sum->status, kErrCount);
+      const int cnt = static_cast<int>(want < kCap ? want : kCap);  // staging bounds every access
+      if (lane == 0 && want > kCap) atomicOr(&p.sum->status, kErrCount);
       const uint32_t* ranks2 = reinterpret_cast<const uint32_t*>(p.ranks + static_cast<int64_t>(row) * kBmrSlots);
       int col[kSteps];
       uint32_t rk2[kSteps / 2];  // ranks of steps q (low half) and q + kSteps / 2 (high half)
@@ -645,7 +653,7 @@ int64_t clamp_grid(int64_t want, int num_sms, int per_sm) {
 template <typename T, int LOGW, int G>
 void launch_bmr_g(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s) {
   if (numeric) {
-    const size_t smem = static_cast<size_t>(kRowsPerCta) * numeric_warp_bytes<T>();
+    const size_t smem = static_cast<size_t>(kRowsPerCta) * numeric_warp_bytes<T, G>();
     static int per_sm = 0;
     if (per_sm == 0) per_sm = occupancy(bmr_numeric_kernel<T, G>, 32 * kRowsPerCta, smem);
     const int64_t per_cta = static_cast<int64_t>(kRowsPerCta) * kHdrRows;
