@@ -1,5 +1,6 @@
 // Heavy rows: rows with too many products for the one-warp workspaces.  One
-// CTA owns one row (the shard pattern of Sec. 4), so every output segment is
+// CTA owns one row, or one (row, column slice) item of a row with many
+// stored entries (the shard pattern of Sec. 4), so every output segment is
 // written by one CTA and no CTA waits on another.
 //
 // Dense rows (kClsRcd): the row's column range is at most 65,536 columns and
@@ -15,7 +16,10 @@
 //             previous slice stopped) and add a * b into the dense value
 //             window with shared-memory atomics (the atomic level of Sec. 4).
 //             The flags of the slice are then scanned in column order, so the
-//             slice's entries are written sorted.
+//             slice's entries are written sorted.  A row whose output fits
+//             one or two windows indexes the window by output rank instead
+//             (a bitmap of its columns and word ranks; rcd_compact_row) and
+//             needs no slices.
 //
 // Wide rows (kClsWb): column range up to 2^20 columns.  A bitmap over the
 // whole range (one bit per column) is the workspace:
