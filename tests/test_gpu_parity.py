@@ -322,6 +322,30 @@ def test_handle_reuse_and_growth():
     assert_matches_oracle(A2, B, rowptr, colidx, vals)
 
 
+@pytest.mark.parametrize("dtype", DTYPES)
+@pytest.mark.parametrize("shift", [0, 1, 3])
+def test_output_arrays_at_any_alignment(dtype, shift):
+    """C's column and value arrays given at an offset of `shift` elements (not
+    16-byte aligned unless shift is 0): the register-bitmap rows, copied out
+    in 16-byte groups when both arrays are aligned, must give the same C."""
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, SpGEMM
+    rng = np.random.default_rng(35)
+    A = uniform_csr(5000, 3000, 12, rng, dtype, "sym")   # 12 entries per row
+    B = uniform_csr(3000, 40_000, 30, rng, dtype, "sym")  # 30 per row: 32-lane groups, ~360 entries per C row
+    dA, dB = DeviceCSR.from_host(A), DeviceCSR.from_host(B)
+    tdt = torch.float32 if dtype == np.float32 else torch.float64
+    with SpGEMM(dA, dB) as op:
+        nnz = op.symbolic()
+        ci = torch.empty(nnz + shift, dtype=torch.int32, device="cuda")[shift:]
+        cv = torch.empty(nnz + shift, dtype=tdt, device="cuda")[shift:]
+        C = op.numeric(out=DeviceCSR(A.nrows, B.ncols, op.c_rowptr, ci, cv))
+        op.wait()
+        info = op.plan_info()
+        rowptr, colidx, vals = C.to_host()
+    assert info["bitmap_rows"] == A.nrows
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
 def test_many_live_handles():
     """More live products than one block of recycled pinned summaries (64):
     each of 150 open SpGEMM objects keeps its own summary and result, and
