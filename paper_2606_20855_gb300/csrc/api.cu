@@ -152,6 +152,7 @@ struct Plan {
   int64_t* ew_chunk_begin = nullptr;
   int32_t* ew_chunk_row = nullptr;
   int64_t* ew_chunk_off = nullptr;
+  int64_t* ew_chunk_split = nullptr;
   int64_t* ew_partials = nullptr;
   int32_t* rcd_scnt = nullptr;
   int32_t* rcd_mega = nullptr;
@@ -557,6 +558,7 @@ ws_status_t carve_ewise(Plan* pl, int64_t m, int64_t nc_max, cudaStream_t s) {
   const size_t o_begin = off; off = align_up(off + 8 * static_cast<size_t>(m + 1), 256);
   const size_t o_row = off; off = align_up(off + 4 * static_cast<size_t>(nc_max), 256);
   const size_t o_off = off; off = align_up(off + 8 * static_cast<size_t>(nc_max + 1), 256);
+  const size_t o_split = off; off = align_up(off + 8 * static_cast<size_t>(nc_max), 256);
   const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
   ws_status_t st = pl->ew.reserve(off, s);
   if (st != WS_OK) return st;
@@ -565,6 +567,7 @@ ws_status_t carve_ewise(Plan* pl, int64_t m, int64_t nc_max, cudaStream_t s) {
   pl->ew_chunk_begin = reinterpret_cast<int64_t*>(b + o_begin);
   pl->ew_chunk_row = reinterpret_cast<int32_t*>(b + o_row);
   pl->ew_chunk_off = reinterpret_cast<int64_t*>(b + o_off);
+  pl->ew_chunk_split = reinterpret_cast<int64_t*>(b + o_split);
   pl->ew_partials = reinterpret_cast<int64_t*>(b + o_part);
   return WS_OK;
 }
@@ -581,6 +584,7 @@ EwisePlan<T> make_ewise(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, const
   p.chunk_begin = pl->ew_chunk_begin;
   p.chunk_row = pl->ew_chunk_row;
   p.chunk_off = pl->ew_chunk_off;
+  p.chunk_split = pl->ew_chunk_split;
   p.nc_max = pl->ew_nc_max;
   p.partials = pl->ew_partials;
   p.sum = pl->dsum;

@@ -8,8 +8,9 @@
 //
 // Work units.  Row i is seen as the merge of its two sorted column lists
 // (length na_i + nb_i) and cut into chunks of `diag` merged positions
-// (merge-path diagonals; an empty row has none).  A chunk boundary is placed by a binary search on the two
-// lists, with the entry of A ahead of an equal entry of B and an equal pair
+// (merge-path diagonals; an empty row has none).  A chunk boundary is placed
+// by a binary search on the two lists, with the entry of A ahead of an equal
+// entry of B and an equal pair
 // never cut apart, so every chunk is the merge of a contiguous part of each
 // list and no position of C is produced by two chunks.  Chunks balance long
 // rows (power-law graphs) across the GPU.
@@ -25,9 +26,11 @@
 // at least one full window unless a list is exhausted.
 //
 // Symbolic pass: chunks per row -> scan -> chunk -> row map -> count per
-// chunk -> scan (chunk output offsets, nnz(C)) -> C.rowptr[i] = offset of the
-// first chunk of row i (of the next chunk for an empty row).  Numeric pass: every chunk merges again and writes its
-// entries from its offset.
+// chunk (the chunk's split, found by the binary search, is kept) -> scan
+// (chunk output offsets, nnz(C)) -> C.rowptr[i] = offset of the first chunk
+// of row i (of the next chunk for an empty row).  Numeric pass: every chunk
+// reads its split and the next chunk's, merges again and writes its entries
+// from its offset.
 #include <climits>
 
 #include "ws_internal.cuh"
@@ -252,6 +255,34 @@ __device__ int64_t merge_seq(const int32_t* a, const T* va, int64_t na, const in
   return out;
 }
 
+// The chunk's ranges a[i0..i1) and b[j0..j1) (merged positions d0..d1 of
+// the row).  The symbolic pass finds the split at d0 by binary search and
+// keeps it in chunk_split as 2 * i0 + (j0 - (d0 - i0)) (an equal pair
+// straddling the cut puts j0 one past d0 - i0); the numeric pass reads its
+// own and the next chunk's split from there, clamped to the lists (if the
+// input changed in between, the ranges stay inside them and the count check
+// reports it).
+template <bool FILL, typename T>
+__device__ __forceinline__ void chunk_bounds(const EwisePlan<T>& p, int64_t c, const int32_t* a, int64_t na,
+                                             const int32_t* b, int64_t nb, int64_t d0, int64_t d1, int64_t* i0,
+                                             int64_t* j0, int64_t* i1, int64_t* j1) {
+  auto decode = [&](int64_t d, int64_t code, int64_t* i, int64_t* j) {
+    const int64_t lo = d - nb > 0 ? d - nb : 0, hi = d < na ? d : na;
+    const int64_t x = code >> 1;
+    *i = x < lo ? lo : (x > hi ? hi : x);
+    const int64_t y = d - *i + (code & 1);
+    *j = y > nb ? nb : y;
+  };
+  if constexpr (!FILL) {
+    if (d0 > 0) merge_split(a, na, b, nb, d0, i0, j0);
+    if (d1 < na + nb) merge_split(a, na, b, nb, d1, i1, j1);
+    if (threadIdx.x % p.group == 0) p.chunk_split[c] = 2 * *i0 + (*j0 - (d0 - *i0));
+  } else {
+    decode(d0, p.chunk_split[c], i0, j0);
+    if (d1 < na + nb) decode(d1, p.chunk_split[c + 1], i1, j1);  // the next chunk belongs to this row
+  }
+}
+
 // One thread per chunk, same contract as ew_merge_kernel.
 template <typename T, int OP, bool FILL>
 __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(const EwisePlan<T> p) {
@@ -274,8 +305,7 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(
     const int64_t d0 = k * p.diag;
     const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
     int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
-    if (d0 > 0) merge_split(a, na, b, nb, d0, &i0, &j0);
-    if (d1 < na + nb) merge_split(a, na, b, nb, d1, &i1, &j1);
+    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1);
     if constexpr (FILL) {
       const int64_t o0 = p.chunk_off[c];
       const int64_t cap = p.chunk_off[c + 1] - o0;
@@ -336,8 +366,7 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_kernel(cons
     const int64_t d0 = k * p.diag;
     const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
     int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
-    if (d0 > 0) merge_split(a, na, b, nb, d0, &i0, &j0);
-    if (d1 < na + nb) merge_split(a, na, b, nb, d1, &i1, &j1);
+    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1);
     if constexpr (FILL) {
       const int64_t o0 = p.chunk_off[c];
       const int64_t cap = p.chunk_off[c + 1] - o0;

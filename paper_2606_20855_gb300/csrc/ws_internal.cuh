@@ -176,6 +176,7 @@ struct EwisePlan {
   int64_t* chunk_begin;  // [m + 1]: first chunk of each row (chunks per row, then scanned in place)
   int32_t* chunk_row;    // [nc_max]: row of each chunk
   int64_t* chunk_off;    // [nc_max + 1]: C offset of each chunk (counts, then scanned in place)
+  int64_t* chunk_split;  // [nc_max]: 2 * (A entries before the chunk) + (1 if an equal pair straddles its start)
   int64_t nc_max;        // bound on the number of chunks: m + (nnz(A) + nnz(B)) / diag + 1
   int64_t* partials;     // scan scratch for max(m, nc_max) entries
   DevSummary* sum;
