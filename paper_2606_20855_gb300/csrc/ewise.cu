@@ -255,6 +255,71 @@ __device__ int64_t merge_seq(const int32_t* a, const T* va, int64_t na, const in
   return out;
 }
 
+// SpAdd fill of one chunk: every merge step emits one entry of the union,
+// so after a scalar head up to the first 16-byte boundary of C the steps go
+// four at a time into registers with fixed slots and leave as one 16-byte
+// store of columns and one (fp32) or two (fp64) of values; the tail is
+// scalar again.  `cap` is the chunk's entry count from the symbolic pass.
+template <typename T>
+__device__ int64_t merge_add_fill(const int32_t* a, const T* va, int64_t na, const int32_t* b, const T* vb,
+                                  int64_t nb, int32_t* c, T* v, int64_t cap, int64_t abs0, bool vec, bool* bad) {
+  int64_t i = 0, j = 0, n = 0;
+  int ca = na > 0 ? a[0] : INT_MAX;
+  int cb = nb > 0 ? b[0] : INT_MAX;
+  // One merge step: the smaller head (both when equal, values added).
+  auto step = [&](int* col, T* val) {
+    const bool take_a = ca <= cb, take_b = cb <= ca;
+    *col = take_a ? ca : cb;
+    const T x = take_a ? va[i] : T(0);
+    const T y = take_b ? vb[j] : T(0);
+    *val = take_a ? (take_b ? x + y : x) : y;
+    if (take_a) {
+      ++i;
+      ca = i < na ? a[i] : INT_MAX;
+    }
+    if (take_b) {
+      ++j;
+      cb = j < nb ? b[j] : INT_MAX;
+    }
+  };
+  auto more = [&]() { return i < na || j < nb; };
+  if (vec) {
+    for (int h = 0; h < 3 && more() && n < cap && ((abs0 + n) & 3); ++h, ++n) step(c + n, v + n);
+    for (int64_t g = 0; g < (na + nb) / 4 + 1 && n + 4 <= cap; ++g, n += 4) {
+      int c0, c1, c2, c3;
+      T v0, v1, v2, v3;
+      // n + 4 <= cap: four more entries exist unless the lists changed since the count
+      if (!more()) break;
+      step(&c0, &v0);
+      if (!more()) { *bad = true; break; }
+      step(&c1, &v1);
+      if (!more()) { *bad = true; break; }
+      step(&c2, &v2);
+      if (!more()) { *bad = true; break; }
+      step(&c3, &v3);
+      *reinterpret_cast<int4*>(c + n) = make_int4(c0, c1, c2, c3);
+      if constexpr (sizeof(T) == 4) {
+        *reinterpret_cast<float4*>(v + n) = make_float4(v0, v1, v2, v3);
+      } else {
+        reinterpret_cast<double2*>(v + n)[0] = make_double2(v0, v1);
+        reinterpret_cast<double2*>(v + n)[1] = make_double2(v2, v3);
+      }
+    }
+  }
+  for (int64_t guard = 0; guard <= na + nb && more(); ++guard, ++n) {
+    int col;
+    T val;
+    step(&col, &val);
+    if (n < cap) {
+      c[n] = col;
+      v[n] = val;
+    } else {
+      *bad = true;
+    }
+  }
+  return n;
+}
+
 // The chunk's ranges a[i0..i1) and b[j0..j1) (merged positions d0..d1 of
 // the row).  The symbolic pass finds the split at d0 by binary search and
 // keeps it in chunk_split as 2 * i0 + (j0 - (d0 - i0)) (an equal pair
@@ -309,9 +374,15 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(
     if constexpr (FILL) {
       const int64_t o0 = p.chunk_off[c];
       const int64_t cap = p.chunk_off[c + 1] - o0;
-      SeqWriter<T> w(p.c_colidx + o0, p.c_vals + o0, cap, o0, vec);
-      const int64_t n = merge_seq<T, OP, true>(a + i0, p.A.vals + a0 + i0, i1 - i0, b + j0, p.B.vals + b0 + j0,
-                                               j1 - j0, &w, &bad);
+      int64_t n;
+      if constexpr (OP == kEwiseAdd) {
+        n = merge_add_fill<T>(a + i0, p.A.vals + a0 + i0, i1 - i0, b + j0, p.B.vals + b0 + j0, j1 - j0,
+                              p.c_colidx + o0, p.c_vals + o0, cap, o0, vec, &bad);
+      } else {
+        SeqWriter<T> w(p.c_colidx + o0, p.c_vals + o0, cap, o0, vec);
+        n = merge_seq<T, OP, true>(a + i0, p.A.vals + a0 + i0, i1 - i0, b + j0, p.B.vals + b0 + j0, j1 - j0, &w,
+                                   &bad);
+      }
       if (n != cap) bad = true;
     } else {
       p.chunk_off[c + 1] = merge_seq<T, OP, false>(a + i0, nullptr, i1 - i0, b + j0, nullptr, j1 - j0, nullptr, &bad);
