@@ -107,7 +107,10 @@ ws_status_t ws_csr_create(ws_csr_t* out, int64_t nrows, int64_t ncols, int64_t n
  * the caller needs nnz(C) to allocate C's arrays.  The row plan (row classes,
  * per-row workspaces) is kept in C's handle for ws_spgemm_numeric.
  * Device scratch is allocated stream-ordered on `stream` and cached in C's
- * handle across calls.
+ * handle across calls.  The first call on a device sets the release
+ * threshold of that device's default stream-ordered memory pool to its
+ * maximum, so memory freed by destroyed handles stays in the pool for the
+ * next ones (it is returned to the system when the process exits).
  */
 ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_out, ws_stream_t stream);
 
@@ -215,7 +218,9 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream);
 /*
  * ws_csr_destroy -- releases the handle and the scratch it owns (never the
  * borrowed arrays).  NULL-safe.  Synchronises the device if the handle owns
- * scratch, so pending work that uses it completes first.
+ * scratch, so pending work that uses it completes first; device scratch goes
+ * back to the stream-ordered pool and the pinned host summary to a
+ * process-wide free list.
  */
 ws_status_t ws_csr_destroy(ws_csr_t handle);
 
