@@ -300,11 +300,12 @@ __device__ __forceinline__ void rcd_warp_add(const RowPlan<T>& p, T* dense, uint
 //      pieces of kRcdPiece entries (scan of the piece counts into e_pp);
 //   2. the warps share the pieces and set the bit of every product column;
 //   3. each thread ranks four consecutive bitmap words (one barrier for
-//      the CTA scan) and keeps the rank of every word (uint16); after a
-//      barrier each thread writes the column indices of four words strided
-//      by the CTA size (a dense stretch of columns is shared out);
+//      the CTA scan) and keeps the rank of every word (uint16);
 //   4. the warps take the pieces again and add a * b at the rank of each
-//      column (shared-memory atomics);
+//      column (shared-memory atomics); the product that set a column's bit
+//      in step 2 (its flag is kept per piece and lane) writes the column
+//      index of C there (rows with too many pieces for the flags write the
+//      column indices from the bitmap in step 3 instead);
 //   5. the window is copied to C's values with coalesced stores and cleared;
 //      after the last pass every thread clears its bitmap words.
 // All threads of the CTA call it; the caller's barrier follows.  Returns
@@ -312,6 +313,7 @@ __device__ __forceinline__ void rcd_warp_add(const RowPlan<T>& p, T* dense, uint
 // multi-pass row would cost more than column slices.
 constexpr int kRcdPiece = 256;  // B entries of one warp-sized piece
 constexpr int kCompactPre = 6400;  // byte offset of the word ranks in the entry cache
+constexpr int kCompactFresh = kCompactPre + kMaxBitmapSpan / 32 * 2;  // byte offset of the fresh flags
 constexpr int kCompactPasses = 2;  // value windows a compact row may take
 constexpr long long kCompactExtraProducts = 65536;  // products re-walked by the extra passes, at most
 
@@ -327,6 +329,12 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
   int* e_pp = reinterpret_cast<int*>(cache + kRcdMegaA * 16);         // first piece of every entry
   int* e_len = e_pp + kRcdMegaA + 1;                                  // B row lengths
   uint16_t* pre = reinterpret_cast<uint16_t*>(cache + kCompactPre);  // rank of every bitmap word
+  // Per piece and lane, which of the lane's products set its column's bit
+  // first (one byte: bit u for the product at u * 32 + lane of the piece).
+  // That product writes the column index of C in step 4; a row with more
+  // pieces than the array holds writes them from the bitmap in step 3.
+  uint8_t* fresh = cache + kCompactFresh;
+  const int cache_bytes = kRcdCacheA * static_cast<int>(2 * sizeof(long long) + sizeof(T) + sizeof(int));
   uint32_t* bm = reinterpret_cast<uint32_t*>(flags);
   const int nnz = static_cast<int>(cend - cbase);
   // 1. entries and pieces
@@ -374,6 +382,7 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
   }
   __syncthreads();
   const int npieces = s_work[0];
+  const bool by_fresh = static_cast<long long>(npieces) * 32 <= cache_bytes - kCompactFresh;
   // Every window pass after the first walks all products again; past the
   // budget the column-sliced path (one walk) is cheaper.
   const int passes = (nnz + width - 1) / width;
@@ -395,17 +404,20 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
     int cc[kRcdPiece / 32];
 #pragma unroll
     for (int u = 0; u < kRcdPiece / 32; ++u) cc[u] = t0 + u * 32 < e ? p.B.colidx[b + t0 + u * 32] : -1;
+    uint32_t first = 0;
 #pragma unroll
     for (int u = 0; u < kRcdPiece / 32; ++u) {
       const long long off = cc[u] - lo;
       if (cc[u] >= 0) {
         if (off >= 0 && off <= hi - lo) {
-          atomicOr(bm + (off >> 5), 1u << (off & 31));
+          const uint32_t bit = 1u << (off & 31);
+          if ((atomicOr(bm + (off >> 5), bit) & bit) == 0u) first |= 1u << u;
         } else {
           *bad = true;
         }
       }
     }
+    if (by_fresh) fresh[pc * 32 + lane] = static_cast<uint8_t>(first);
   }
   __syncthreads();
   // 3. word ranks and C's column indices; thread t owns the bitmap words
@@ -437,10 +449,11 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
     run += __popc(wv[q]);
   }
   __syncthreads();
-  // Column indices in order: thread t writes those of the words t, t + 512,
-  // t + 1024, t + 1536 (strided, so a dense stretch of columns is shared out).
+  // Rows with too many pieces for the fresh flags: column indices in order,
+  // thread t writing those of the words t, t + 512, t + 1024, t + 1536
+  // (strided, so a dense stretch of columns is shared out).
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
+  for (int q = 0; q < 4 && !by_fresh; ++q) {
     const int w = q * kRcdNumThreads + threadIdx.x;
     const long long col0 = lo + (static_cast<long long>(w) << 5) - 1;
     int at = pre[w];
@@ -473,13 +486,17 @@ __device__ bool rcd_compact_row(const RowPlan<T>& p, T* dense, uint8_t* flags, u
         cc[u] = t < e ? p.B.colidx[b + t] : -1;
         bv[u] = t < e ? p.B.vals[b + t] : T(0);
       }
+      const uint32_t first = by_fresh ? fresh[pc * 32 + lane] : 0u;
 #pragma unroll
       for (int u = 0; u < kRcdPiece / 32; ++u) {
         const long long off = cc[u] - lo;
         if (cc[u] >= 0 && off >= 0 && off <= hi - lo) {
           const int w = static_cast<int>(off >> 5);
           const int rank = pre[w] + __popc(bm[w] & ((1u << (off & 31)) - 1u)) - q0;
-          if (rank >= 0 && rank < width) atomicAdd(dense + rank, av * bv[u]);
+          if (rank >= 0 && rank < width) {
+            atomicAdd(dense + rank, av * bv[u]);
+            if ((first >> u) & 1u) p.c_colidx[cbase + q0 + rank] = cc[u];
+          }
         }
       }
     }
