@@ -117,11 +117,16 @@ __global__ void __launch_bounds__(kRcdThreads, 3) rcd_symbolic_kernel(const RowP
     long long cnt = 0;
     const int n16 = (span + 15) >> 4;
     constexpr int kChunksPerSlice = kRcdWidthBytes / static_cast<int>(sizeof(T)) / 16;
-    for (int i = threadIdx.x; i < n16; i += kRcdThreads) {
-      const int n = nonzero_bytes(flags4[i]);
+    static_assert(kChunksPerSlice % 32 == 0, "a warp's 32 chunks lie in one slice");
+    // Lane l of warp w reads chunk i0 + l; the warp's chunks share one slice,
+    // so their counts are summed in the warp and added with one atomic.
+    for (int i0 = threadIdx.x & ~31; i0 < n16; i0 += kRcdThreads) {
+      const int i = i0 + (threadIdx.x & 31);
+      const int n = i < n16 ? nonzero_bytes(flags4[i]) : 0;
       cnt += n;
-      if (n) atomicAdd(&s_slice[i / kChunksPerSlice], n);
-      flags4[i] = make_uint4(0u, 0u, 0u, 0u);
+      const int wsum = __reduce_add_sync(kFull, n);
+      if ((threadIdx.x & 31) == 0 && wsum) atomicAdd(&s_slice[i0 / kChunksPerSlice], wsum);
+      if (i < n16) flags4[i] = make_uint4(0u, 0u, 0u, 0u);
     }
     long long total;
     block_exclusive_scan(cnt, s_scan, &total);
