@@ -255,7 +255,7 @@ constexpr size_t numeric_warp_bytes() {
 }
 
 template <typename T, int G>
-__global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_numeric_kernel(const RowPlan<T> p) {
+__global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_numeric_kernel(const RowPlan<T> p, int hb) {
   constexpr int kGroups = 32 / G;
   constexpr int kSteps = kBmrMaxA / kGroups;
   constexpr int kEnt = kHdrRows * kBmrMaxA;
@@ -276,15 +276,16 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
   long long* h_cnt = h_cbase + kHdrRows;
   int* h_row = reinterpret_cast<int*>(h_cnt + kHdrRows);
 
+  // hb (1..kHdrRows) rows per batch: fewer when the segment is too short to
+  // give every warp of the grid a full batch.
   const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
-  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * kHdrRows; r0 < p.seg_len;
-       r0 += warps * kHdrRows) {
-    // Batch header: lane i < kHdrRows fetches row r0 + i.
+  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * hb; r0 < p.seg_len; r0 += warps * hb) {
+    // Batch header: lane i < hb fetches row r0 + i.
     int na_l = 0;
     long long ra_l = 0;
     if (lane < kHdrRows) {
       int row_l = -1;
-      if (r0 + lane < p.seg_len) {
+      if (lane < hb && r0 + lane < p.seg_len) {
         row_l = p.perm ? p.perm[p.seg_begin + r0 + lane] : static_cast<int>(p.seg_begin + r0 + lane);
         ra_l = p.A.rowptr[row_l];
         const long long na = p.A.rowptr[row_l + 1] - ra_l;
@@ -656,9 +657,14 @@ void launch_bmr_g(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s
     const size_t smem = static_cast<size_t>(kRowsPerCta) * numeric_warp_bytes<T, G>();
     static int per_sm = 0;
     if (per_sm == 0) per_sm = occupancy(bmr_numeric_kernel<T, G>, 32 * kRowsPerCta, smem);
-    const int64_t per_cta = static_cast<int64_t>(kRowsPerCta) * kHdrRows;
+    // Rows per warp batch: kHdrRows, unless that leaves warps of one full
+    // wave idle (a short segment), then as few as one.
+    const int64_t wave_warps = static_cast<int64_t>(num_sms) * per_sm * kRowsPerCta;
+    int64_t hb = (p.seg_len + wave_warps - 1) / wave_warps;
+    hb = hb < 1 ? 1 : (hb > kHdrRows ? kHdrRows : hb);
+    const int64_t per_cta = static_cast<int64_t>(kRowsPerCta) * hb;
     const int64_t grid = clamp_grid((p.seg_len + per_cta - 1) / per_cta, num_sms, per_sm);
-    bmr_numeric_kernel<T, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
+    bmr_numeric_kernel<T, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p, static_cast<int>(hb));
     return;
   }
   const size_t smem = static_cast<size_t>(kRowsPerCta) * BmrShape<LOGW>::bytes();
