@@ -58,8 +58,8 @@ NOMINAL_HBM_GBS = 8000.0
 # rows, so traffic grows in proportion).  Symbolic: bmr_plan_kernel only (the
 # analysis, scatter and scan kernels move a few MB).  Valid only for the
 # kernels they were taken on.
-NUMERIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.415403e9 + 1.019798e9)}
-SYMBOLIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.027999e9 + 0.218566e9)}
+NUMERIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.408874e9 + 1.017987e9)}
+SYMBOLIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.028002e9 + 0.218672e9)}
 
 
 def products_per_row(A, B) -> np.ndarray:
