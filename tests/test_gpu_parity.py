@@ -11,6 +11,7 @@ import torch
 
 from synth import HostCSR, random_csr, rmat_pattern, uniform_csr
 from tests._gpu import assert_matches_oracle, run_gpu, tuning
+from tests._helpers import TOL
 
 pytestmark = pytest.mark.gpu
 
@@ -214,6 +215,28 @@ def test_dense_rows_slice_parts(dtype):
     assert info["rcd_rows"] >= 38
     assert np.diff(rowptr)[5] == slice_w and np.diff(rowptr)[6] == slice_w + 1
     assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_dense_rows_many_products_few_columns(dtype):
+    """Dense heavy rows with far more products than output entries: 200
+    stored entries whose B rows (1000 entries each) share a pool of 6000
+    columns, so 200,000 products fall on at most 6000 outputs.  The output fits
+    one value window, but the products are too many for the per-piece first
+    flags, so the column indices come from the bitmap walk instead."""
+    rng = np.random.default_rng(36)
+    n = 1 << 16
+    pool = rng.choice(n, size=6000, replace=False)
+    k = 260
+    rows = {i: rng.choice(pool, size=1000, replace=False).tolist() for i in range(k)}
+    B = _csr(k, n, rows, dtype=dtype)
+    B.vals = (2 * rng.random(B.nnz) - 1).astype(dtype)
+    arows = {i: rng.choice(k, size=200, replace=False).tolist() for i in range(6)}
+    A = _csr(6, k, arows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["rcd_rows"] == 6
+    assert assert_matches_oracle(A, B, rowptr, colidx, vals) <= TOL[np.dtype(dtype)]
 
 
 @pytest.mark.parametrize("dtype", DTYPES)
