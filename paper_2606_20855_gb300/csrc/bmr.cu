@@ -104,27 +104,6 @@ __device__ __forceinline__ void load_products(const RowPlan<T>& p, int64_t ra, i
   }
 }
 
-// Sets the bit of every product column; returns how many bits were 0 before
-// (when COUNT).  The caller clears the words after its last use.
-template <class S, bool COUNT, int kSteps>
-__device__ __forceinline__ int set_bits(uint32_t* bm, const int* col, int lo) {
-  int fresh = 0;
-#pragma unroll
-  for (int s = 0; s < kSteps; ++s) {
-    if (col[s] >= 0) {
-      const uint32_t off = static_cast<uint32_t>(col[s] - lo);
-      const uint32_t bit = 1u << (off & 31u);
-      uint32_t* word = bm + phys_word<S>(off >> 5);
-      if constexpr (COUNT) {
-        fresh += (atomicOr(word, bit) & bit) == 0u;
-      } else {
-        atomicOr(word, bit);
-      }
-    }
-  }
-  return fresh;
-}
-
 template <class S, int kSteps>
 __device__ __forceinline__ void clear_bits(uint32_t* bm, const int* col, int lo) {
 #pragma unroll
