@@ -91,6 +91,11 @@ typedef enum {
  *            WS_ERR_INVALID_CSR and no handle.  Pass 0 for an output handle.
  *   stream   stream for the validation kernel
  * The handle owns only library scratch (released by ws_csr_destroy).
+ * Passage: the compressed-format invariants of Sec. 1 ("Complex Data
+ * Structure Invariants": CSR is prefix sums over contiguous buffers) and
+ * Sec. 3.1 (position arrays are cumulative sums that must stay monotonically
+ * non-decreasing); validation checks exactly those plus sorted, in-range
+ * column indices.
  */
 ws_status_t ws_csr_create(ws_csr_t* out, int64_t nrows, int64_t ncols, int64_t nnz, int64_t* rowptr,
                           int32_t* colidx, void* vals, ws_dtype_t dtype, int validate,
@@ -111,6 +116,11 @@ ws_status_t ws_csr_create(ws_csr_t* out, int64_t nrows, int64_t ncols, int64_t n
  * threshold of that device's default stream-ordered memory pool to its
  * maximum, so memory freed by destroyed handles stays in the pool for the
  * next ones (it is returned to the system when the process exits).
+ * Passage: Sec. 5.1 (Gustavson's SpGEMM, parallel over output fibers: the
+ * count of row i is the number of distinct fibers that row's worker will
+ * write under the shard level) and the `declare` step of the lifecycle in
+ * Sec. 4 ("Building on Finch": the output is initialised and sized before it
+ * is updated).
  */
 ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_out, ws_stream_t stream);
 
@@ -122,6 +132,10 @@ ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_
  * unchanged since).  Asynchronous: work is queued on `stream` and the call
  * returns without waiting; device-side failures are reported by
  * ws_spgemm_wait.  The two arrays are recorded in C's handle.
+ * Passage: Sec. 5.1 (Gustavson's loop: w[j] += A[i,k] * B[k,j] in a per-row
+ * workspace, then row i of C is written from w in sorted column order) and
+ * the `update` -> `freeze` steps of Sec. 4 (the pass updates C's disjoint row
+ * segments and leaves C in read mode).
  */
 ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
                               ws_stream_t stream);
@@ -221,6 +235,9 @@ ws_status_t ws_spgemm_wait(ws_csr_t C, ws_stream_t stream);
  * scratch, so pending work that uses it completes first; device scratch goes
  * back to the stream-ordered pool and the pinned host summary to a
  * process-wide free list.
+ * Passage: the end of the lifecycle of Sec. 4 ("Building on Finch"): once C is
+ * frozen, the workspaces the passes declared are no longer needed.  The
+ * paper has no explicit release call; this one frees the library's share.
  */
 ws_status_t ws_csr_destroy(ws_csr_t handle);
 
@@ -293,8 +310,12 @@ ws_status_t ws_set_tuning(int key, int64_t value);
  * Scratch lives in a fixed array compiled into the library (about 33 KB),
  * which every GPU that loads the library keeps until the process exits.  The
  * call itself calls no cudaMalloc, cudaFree or other allocating routine.
- * The first call on a device looks up that array's device address; make
- * that first call before any stream capture.  All calls share the array:
+ * The first call on a device looks up that array's device address and
+ * keeps it for the life of the process; make that first call before any
+ * stream capture, and do not call this function again on a device after
+ * cudaDeviceReset (or anything else that destroys the device's primary
+ * context), because the kept address then names freed memory.  All calls
+ * share the array:
  * calls that may run at the same time on the GPU (on unordered streams) race
  * and give wrong results.  Returns WS_ERR_INVALID_ARG for a NULL rowptr or a
  * negative nrows, WS_ERR_CUDA if a CUDA call fails.

@@ -41,7 +41,9 @@ int64_t* g_scratch_ptr[kMaxDevices] = {};
 
 // Device address of the fixed scratch on the current device.  The first call
 // on a device looks it up (cudaGetSymbolAddress, with that device current)
-// and remembers it.
+// and remembers it for the life of the process.  A cudaDeviceReset destroys
+// the module that holds the array, so the remembered address is not valid
+// after one; the header says not to call the entry point across a reset.
 cudaError_t static_scratch(int dev, int64_t** out) {
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
