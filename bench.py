@@ -3,25 +3,34 @@
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
 A step is one full product -- symbolic pass (including its nnz read-back),
-allocation of C, numeric pass and the final status read -- over device-
-resident inputs.  Between timed steps the L2 is flushed by writing a buffer
-larger than it; each step is timed with CUDA events on the stream the
-library runs on.  Throughput is GFLOP/s = 2 x products / time; the
-effective HBM bandwidth uses the compulsory bytes (read A and B once, write
-C once, at their stored widths).
+a fresh allocation of C's arrays, numeric pass and the final status read --
+over device-resident inputs.  Between timed steps the L2 is flushed by
+writing a buffer larger than it; each step is timed with CUDA events on the
+stream the library runs on.  Throughput is GFLOP/s = 2 x products / time;
+the effective HBM bandwidth uses the compulsory bytes (read A and B once,
+write C once, at their stored widths).
+
+The headline is the uniform 2^20 x 2^16 (16/row) times 2^16 x 2^16 (32/row)
+product in fp32.  Without --workload, the line also carries `per_config`:
+the same measurement (value, roofline, end to end, CPU oracle, clocks) for
+each of the five named SpGEMM workloads, each timed for at least half a
+second, and `sustained`: the headline product timed again over at least one
+second with its own clock record.
 
 Extra keys: `e2e` (the same product through the public Python API from
 pinned host inputs to the host copy of C, copies inside the timed region),
+`roofline` (the whole product -- symbolic + numeric, the span the throughput
+target is set on -- against the measured copy bandwidth, with each pass's own
+figure under `passes`; `traffic` is the DRAM bytes ncu recorded for the
+current kernel sources, null when none match), `cpu_baseline` (the CPU oracle
+on a bounded row sample, on this host's cores), `clocks` (nvidia-smi samples
+during the timed region).
+
 With an elementwise workload (``--workload ewise_* --op add|mul``) a step is
 one elementwise operation C = A + B or C = A .* B and the value is its
 effective bandwidth in GB/s of compulsory bytes; with ``--workload spmspv_*``
 a step is one sparse matrix - sparse vector product y = A x (A resident by
 columns, x the step's input), also in GB/s of compulsory bytes.
-
-`roofline` (the whole product -- symbolic + numeric, the span the throughput
-target is set on -- against the measured copy bandwidth, with each pass's own
-figure under `passes`), `cpu_baseline` (the CPU oracle on a bounded row sample, on
-this host's cores), `clocks` (nvidia-smi samples during the timed region).
 
 Under torchrun (N > 1) every rank runs its own replica of the workload on its
 own GPU (no collective on the data path); rank 0 prints the line with the
@@ -44,7 +53,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-from synth import EWISE_WORKLOADS, SPMSPV_WORKLOADS, WORKLOADS, ewise_workload, spmspv_workload, workload  # noqa: E402
+from synth import (EWISE_WORKLOADS, SPMSPV_WORKLOADS, WORKLOAD_ORDER, WORKLOADS, ewise_workload,  # noqa: E402
+                   spmspv_workload, workload)
 
 METRIC = "SpGEMM GFLOP/s (2×products) and effective HBM GB/s vs 8 TB/s, per config"
 EWISE_METRIC = "SpAdd / Hadamard effective HBM GB/s (compulsory bytes: read A and B, write C)"
@@ -52,14 +62,43 @@ SPMSPV_METRIC = "SpMSpV effective HBM GB/s (compulsory bytes: read x, the column
 DEFAULT_WORKLOAD = "uniform_rect_1m"
 NOMINAL_HBM_GBS = 8000.0
 
-# DRAM bytes (read + write) per pass at full size, from the ncu capture
-# summarised in profiles/bmr_kernels_uniform_rect_1m_262144rows.md: the
-# 262,144-row cut scaled by 4 to 1,048,576 rows (both passes stream their
-# rows, so traffic grows in proportion).  Symbolic: bmr_plan_kernel only (the
-# analysis, scatter and scan kernels move a few MB).  Valid only for the
-# kernels they were taken on.
-NUMERIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.408874e9 + 1.017987e9)}
-SYMBOLIC_TRAFFIC: dict = {"uniform_rect_1m": 4 * (0.028002e9 + 0.218672e9)}
+# Dominant kernel of each pass on the headline workload (the analysis,
+# scatter and scan kernels move a few MB).
+PASS_KERNELS = {"symbolic": "bmr_plan_kernel", "numeric": "bmr_numeric_kernel"}
+PROFILES = os.path.join(ROOT, "profiles")
+
+
+def source_digest(rel_path: str) -> str | None:
+    """First 16 hex digits of the SHA-256 of a source file of this repository."""
+    import hashlib
+    path = os.path.join(ROOT, rel_path)
+    if not os.path.exists(path):
+        return None
+    with open(path, "rb") as fh:
+        return hashlib.sha256(fh.read()).hexdigest()[:16]
+
+
+def recorded_traffic(workload: str, kernel: str) -> float | None:
+    """DRAM bytes (read + write) of one full-size launch of `kernel` on
+    `workload`, from a `traffic-record:` line of a profile summary under
+    profiles/ (an ncu capture of a row cut, scaled by rows), or None when no
+    record exists or the kernel's source changed since it was taken."""
+    if not os.path.isdir(PROFILES):
+        return None
+    for name in sorted(os.listdir(PROFILES)):
+        if not name.endswith(".md"):
+            continue
+        with open(os.path.join(PROFILES, name)) as fh:
+            for line in fh:
+                if not line.startswith("traffic-record:"):
+                    continue
+                kv = dict(x.split("=", 1) for x in line.split()[1:] if "=" in x)
+                if kv.get("workload") != workload or kv.get("kernel") != kernel:
+                    continue
+                if source_digest(kv.get("source", "")) != kv.get("sha256"):
+                    return None  # stale: the kernel changed since the capture
+                return float(kv["dram_bytes"]) * float(kv["of"]) / float(kv["rows"])
+    return None
 
 
 def products_per_row(A, B) -> np.ndarray:
@@ -495,177 +534,253 @@ def run_outer(args, world, rank, local, pg, A, B, dA, dB, ub, flush, stream, dev
     print(json.dumps(line), flush=True)
 
 
-def run_ours(args, world, rank, local, pg) -> None:
+def time_steps(op, steps, flush, stream, device, world, pg, rank, local):
+    """Times `steps` operations (symbolic with its read-back, a fresh C,
+    numeric), the L2 flushed before each; returns per-step, symbolic and
+    numeric milliseconds, the clock record and the max-over-ranks total."""
     import torch
-    from paper_2606_20855_gb300 import _abi
-    from paper_2606_20855_gb300.spgemm import DeviceCSR, Ewise, SpGEMM
-
-    _abi.load()
-    device = torch.device(f"cuda:{local}")
-    torch.cuda.set_device(device)
-    A, B = load_workload(args)
-    same = B is A
-    ew = is_ewise(args)
-    ub = np.zeros(A.nrows, dtype=np.int64) if ew else products_per_row(A, B)
-    products = int(ub.sum())
-    make_op = (lambda x, y: Ewise(x, y, args.op)) if ew else SpGEMM
-    s = 8 if A.vals.dtype == np.float64 else 4
-    stream = torch.cuda.current_stream(device)
-
-    dA = DeviceCSR.from_host(A, device)
-    dB = dA if same else DeviceCSR.from_host(B, device)
-    l2 = torch.cuda.get_device_properties(device).L2_cache_size
-    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
-
-    if args.algo == "outer" and not ew:
-        run_outer(args, world, rank, local, pg, A, B, dA, dB, ub, flush, stream, device)
-        return
-    op = make_op(dA, dB)
-    out = None
-
-    def step():
-        nonlocal out
-        op.symbolic()
-        out = op.numeric(out)
-        op.wait()
-
-    for _ in range(args.warmup):
-        step()
-    nnz = op.nnz
-    info = op.plan_info()
-    algo_bytes = csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz, s)
-    # symbolic pass: read the structure of A and B once, write C.rowptr
-    sym_bytes = csr_bytes(A.nrows, A.nnz, 0) + csr_bytes(B.nrows, B.nnz, 0) + 8 * (A.nrows + 1)
-
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+           torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     clocks = ClockSampler(local).start() if rank == 0 else None
     barrier(world, pg)
     torch.cuda.synchronize(device)
     t_wall0 = time.time()
-    for i in range(args.steps):
+    for i in range(steps):
         flush.fill_(i)  # write > L2 between timed steps (not timed)
         e0, e1, e2 = ev[i]
         e0.record(stream)
         op.symbolic()
         e1.record(stream)
-        out = op.numeric(out)
+        C = op.numeric()  # C's arrays allocated inside the timed span
         e2.record(stream)
         op.wait()
+        del C
     torch.cuda.synchronize(device)
     t_wall1 = time.time()
     barrier(world, pg)
     clk = clocks.stop(t_wall0, t_wall1) if clocks else None
     step_ms = [a.elapsed_time(c) for a, _, c in ev]
-    num_ms = [b.elapsed_time(c) for _, b, c in ev]
     sym_ms = [a.elapsed_time(b) for a, b, _ in ev]
-    total_s = sum(step_ms) / 1e3
-    total_s = reduce_max(total_s, world, pg, device)
-    launches_per_step = info["symbolic_launches"] + info["numeric_launches"]
+    num_ms = [b.elapsed_time(c) for _, b, c in ev]
+    total_s = reduce_max(sum(step_ms) / 1e3, world, pg, device)
+    return step_ms, sym_ms, num_ms, clk, total_s
 
-    # End to end through the public API: pinned host inputs -> device -> product -> host C.
-    e2e = None
-    if args.e2e_steps > 0:
-        hA = [torch.from_numpy(a).pin_memory() for a in (A.rowptr, A.colidx, A.vals)]
-        hB = hA if same else [torch.from_numpy(a).pin_memory() for a in (B.rowptr, B.colidx, B.vals)]
-        h_col = torch.empty(nnz, dtype=torch.int32).pin_memory()
-        h_val = torch.empty(nnz, dtype=hA[2].dtype).pin_memory()
-        h_rp = torch.empty(A.nrows + 1, dtype=torch.int64).pin_memory()
 
-        def e2e_step():
-            tA = DeviceCSR(A.nrows, A.ncols, *[t.to(device, non_blocking=True) for t in hA])
-            tB = tA if same else DeviceCSR(B.nrows, B.ncols, *[t.to(device, non_blocking=True) for t in hB])
-            with make_op(tA, tB) as op2:
-                op2.symbolic()
-                C = op2.numeric()
-                h_rp.copy_(C.rowptr, non_blocking=True)
-                h_col.copy_(C.colidx, non_blocking=True)
-                h_val.copy_(C.vals, non_blocking=True)
-                op2.wait()
-            torch.cuda.synchronize(device)
+def e2e_measure(A, B, make_op, same, device, steps, world, pg, nnz, algo_bytes, ew, products):
+    """The operation through the public Python API from pinned host inputs to
+    the host copy of C, copies inside the timed region."""
+    import torch
+    from paper_2606_20855_gb300.spgemm import DeviceCSR
+    hA = [torch.from_numpy(a).pin_memory() for a in (A.rowptr, A.colidx, A.vals)]
+    hB = hA if same else [torch.from_numpy(a).pin_memory() for a in (B.rowptr, B.colidx, B.vals)]
+    h_col = torch.empty(nnz, dtype=torch.int32).pin_memory()
+    h_val = torch.empty(nnz, dtype=hA[2].dtype).pin_memory()
+    h_rp = torch.empty(A.nrows + 1, dtype=torch.int64).pin_memory()
 
+    def e2e_step():
+        tA = DeviceCSR(A.nrows, A.ncols, *[t.to(device, non_blocking=True) for t in hA])
+        tB = tA if same else DeviceCSR(B.nrows, B.ncols, *[t.to(device, non_blocking=True) for t in hB])
+        with make_op(tA, tB) as op2:
+            op2.symbolic()
+            C = op2.numeric()
+            h_rp.copy_(C.rowptr, non_blocking=True)
+            h_col.copy_(C.colidx, non_blocking=True)
+            h_val.copy_(C.vals, non_blocking=True)
+            op2.wait()
+        torch.cuda.synchronize(device)
+
+    e2e_step()
+    barrier(world, pg)
+    t0 = time.perf_counter()
+    for _ in range(steps):
         e2e_step()
-        barrier(world, pg)
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            e2e_step()
-        e2e_s = reduce_max(time.perf_counter() - t0, world, pg, device)
-        h2d = sum(t.numel() * t.element_size() for t in hA) + (0 if same else sum(t.numel() * t.element_size() for t in hB))
-        d2h = h_rp.numel() * 8 + h_col.numel() * 4 + h_val.numel() * h_val.element_size()
-        e2e_work = algo_bytes if ew else 2.0 * products
-        e2e = {"value": round(e2e_work * args.e2e_steps * world / e2e_s / 1e9, 3), "unit": "GB/s" if ew else "GFLOP/s",
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": args.e2e_steps}
+    e2e_s = reduce_max(time.perf_counter() - t0, world, pg, device)
+    h2d = sum(t.numel() * t.element_size() for t in hA) + (0 if same else sum(t.numel() * t.element_size() for t in hB))
+    d2h = h_rp.numel() * 8 + h_col.numel() * 4 + h_val.numel() * h_val.element_size()
+    work = algo_bytes if ew else 2.0 * float(products)
+    return {"value": round(work * steps * world / e2e_s / 1e9, 3), "unit": "GB/s" if ew else "GFLOP/s",
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
 
+
+def measure(args, name, A, B, steps, warmup, e2e_steps, cpu_s, world, rank, local, pg, min_region_s=0.0,
+            with_traffic=False):
+    """One workload: the timed steps, the roofline of the whole operation and
+    of each pass, end to end and the CPU oracle.  With min_region_s > 0 the
+    step count grows until the timed region lasts at least that long."""
+    import torch
+    from paper_2606_20855_gb300.spgemm import DeviceCSR, Ewise, SpGEMM
+
+    device = torch.device(f"cuda:{local}")
+    stream = torch.cuda.current_stream(device)
+    same = B is A
+    ew = name in EWISE_WORKLOADS
+    ub = np.zeros(A.nrows, dtype=np.int64) if ew else products_per_row(A, B)
+    products = int(ub.sum())
+    make_op = (lambda x, y: Ewise(x, y, args.op)) if ew else SpGEMM
+    s = 8 if A.vals.dtype == np.float64 else 4
+
+    dA = DeviceCSR.from_host(A, device)
+    dB = dA if same else DeviceCSR.from_host(B, device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
+    op = make_op(dA, dB)
+    t0 = time.perf_counter()
+    for _ in range(max(warmup, 1) if min_region_s > 0 else warmup):
+        op.symbolic()
+        C = op.numeric()
+        op.wait()
+        del C
+    torch.cuda.synchronize(device)
+    if min_region_s > 0:  # size the timed region from the warm-up's wall time (slowest rank)
+        per = reduce_max((time.perf_counter() - t0) / max(warmup, 1), world, pg, device)
+        steps = max(steps, min(20000, int(np.ceil(1.2 * min_region_s / max(per, 1e-6)))))
+    nnz = op.nnz
+    info = op.plan_info()
+    algo_bytes = csr_bytes(A.nrows, A.nnz, s) + csr_bytes(B.nrows, B.nnz, s) + csr_bytes(A.nrows, nnz, s)
+    # symbolic pass: read the structure of A and B once, write C.rowptr
+    sym_bytes = csr_bytes(A.nrows, A.nnz, 0) + csr_bytes(B.nrows, B.nnz, 0) + 8 * (A.nrows + 1)
+    step_ms, sym_ms, num_ms, clk, total_s = time_steps(op, steps, flush, stream, device, world, pg, rank, local)
+    launches_per_step = info["symbolic_launches"] + info["numeric_launches"]
     op.close()
+    del op, flush
+    e2e = None
+    if e2e_steps > 0:
+        e2e = e2e_measure(A, B, make_op, same, device, e2e_steps, world, pg, nnz, algo_bytes, ew, products)
+    del dA, dB
+    torch.cuda.empty_cache()
     if rank != 0:
-        return
+        return None
     peaks = measured_peaks()
-    num_mean_s = statistics.mean(num_ms) / 1e3
-
-    def traffic(table):
-        """ncu DRAM bytes for this workload (None: not captured on these kernels, or a row cut)."""
-        if args.rows:
-            return None
-        if table is None:  # whole product: both passes, when both were captured
-            sym, num = traffic(SYMBOLIC_TRAFFIC), traffic(NUMERIC_TRAFFIC)
-            return None if sym is None or num is None else sym + num
-        if table is NUMERIC_TRAFFIC and args.traffic is not None:
-            return args.traffic
-        return table.get(args.workload)
-    eff_gbs = algo_bytes * args.steps * world / total_s / 1e9
-    value = eff_gbs if ew else 2.0 * products * args.steps * world / total_s / 1e9
+    eff_gbs = algo_bytes * steps * world / total_s / 1e9
+    value = eff_gbs if ew else 2.0 * products * steps * world / total_s / 1e9
     base = None
-    if args.cpu_baseline_s > 0:
+    if cpu_s > 0:
         if ew:
             dt, _ = ewise_oracle_timed(A, B, args.op, 1)
             base = {"value": round(algo_bytes / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                     "sample": f"whole operation, {dt:.1f} s, numpy on one core"}
         else:
-            base = cpu_baseline(A, B, ub, args.cpu_baseline_s)
-    line = {
-        "metric": EWISE_METRIC if ew else METRIC,
-        "value": round(value, 3),
-        "unit": "GB/s" if ew else "GFLOP/s",
-        "n_gpus": world,
-        "steps": args.steps,
-        "warmup": args.warmup,
-        "ms_per_step": round(1e3 * total_s / args.steps, 4),
-        "higher_is_better": True,
-        "scaling": "weak",
-        "vs_baseline": None,
+            base = cpu_baseline(A, B, ub, cpu_s)
+    traffic = {"symbolic": None, "numeric": None}
+    if with_traffic and not ew and not args.rows:
+        traffic = {k: recorded_traffic(name, kern) for k, kern in PASS_KERNELS.items()}
+    whole_traffic = (None if traffic["symbolic"] is None or traffic["numeric"] is None
+                     else traffic["symbolic"] + traffic["numeric"])
+    return {
+        "workload": name if not args.rows else f"{name}[:{A.nrows} rows]",
+        "description": EWISE_WORKLOADS[name] if ew else WORKLOADS[name],
+        "value": round(value, 3), "unit": "GB/s" if ew else "GFLOP/s",
+        "ms_per_step": round(1e3 * total_s / steps, 4), "steps": steps, "warmup": warmup,
         "dtype": "f64" if s == 8 else "f32",
-        "data": "synthetic",
-        "config": {
-            "workload": args.workload if not args.rows else f"{args.workload}[:{A.nrows} rows]",
-            "description": EWISE_WORKLOADS[args.workload] if ew else WORKLOADS[args.workload],
-            "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_a": A.nnz, "nnz_b": B.nnz, "nnz_c": int(nnz),
-            **({"op": args.op} if ew else {"products": products}),
-            "l2": "flushed between timed steps (write of a buffer > L2)",
-            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-        },
+        "m": A.nrows, "k": A.ncols, "n": B.ncols, "nnz_a": A.nnz, "nnz_b": B.nnz, "nnz_c": int(nnz),
+        **({"op": args.op} if ew else {"products": products}),
         "effective_hbm_gbs": round(eff_gbs, 1),
         "frac_of_8tbs": round(eff_gbs / NOMINAL_HBM_GBS, 4),
         "phases_ms": {"symbolic_median": round(statistics.median(sym_ms), 4),
                       "numeric_median": round(statistics.median(num_ms), 4),
                       "step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
-        "roofline": dict(roofline_obj(algo_bytes, statistics.mean(step_ms) / 1e3, peaks, traffic(None)),
+        "roofline": dict(roofline_obj(algo_bytes, statistics.mean(step_ms) / 1e3, peaks, whole_traffic),
                          kernel=("whole operation" if ew else "whole product") +
                                 ": symbolic pass (nnz read-back included) + numeric pass",
                          passes={
                              "symbolic": dict(roofline_obj(sym_bytes, statistics.mean(sym_ms) / 1e3, peaks,
-                                                           traffic(SYMBOLIC_TRAFFIC)),
+                                                           traffic["symbolic"]),
                                               kernel="symbolic pass (compulsory bytes: structure of A and B "
                                                      "read once, C.rowptr written)"),
-                             "numeric": dict(roofline_obj(algo_bytes, num_mean_s, peaks, traffic(NUMERIC_TRAFFIC)),
+                             "numeric": dict(roofline_obj(algo_bytes, statistics.mean(num_ms) / 1e3, peaks,
+                                                          traffic["numeric"]),
                                              kernel="numeric pass: " + ("ew_merge_kernel" if ew else
                                                                             numeric_kernels(info))),
                          }),
-        "gpu_launches": int(launches_per_step * args.steps),
+        "gpu_launches": int(launches_per_step * steps),
         "plan": info,
         "clocks": clk,
         "e2e": e2e,
         "cpu_baseline": base,
+        "_total_s": total_s,
     }
+
+
+def run_ours(args, world, rank, local, pg) -> None:
+    import torch
+    from paper_2606_20855_gb300 import _abi
+
+    _abi.load()
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    A, B = load_workload(args)
+    ew = is_ewise(args)
+    if args.algo == "outer" and not ew:
+        from paper_2606_20855_gb300.spgemm import DeviceCSR
+        s_dev = torch.cuda.current_stream(device)
+        l2 = torch.cuda.get_device_properties(device).L2_cache_size
+        flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32, device=device)
+        dA = DeviceCSR.from_host(A, device)
+        dB = dA if B is A else DeviceCSR.from_host(B, device)
+        run_outer(args, world, rank, local, pg, A, B, dA, dB, products_per_row(A, B), flush, s_dev, device)
+        return
+    head = measure(args, args.workload, A, B, args.steps, args.warmup, args.e2e_steps, args.cpu_baseline_s,
+                   world, rank, local, pg, with_traffic=True)
+    # The headline product again over at least one second, with its own clock record.
+    sustained = None
+    if not ew and not args.rows and args.sustained_s > 0:
+        sus = measure(args, args.workload, A, B, args.steps, args.warmup, 0, 0, world, rank, local, pg,
+                      min_region_s=args.sustained_s)
+        if rank == 0:
+            sustained = {"steps": sus["steps"], "ms_per_step": sus["ms_per_step"], "value": sus["value"],
+                         "unit": sus["unit"], "timed_region_s": round(sus["_total_s"], 3), "clocks": sus["clocks"]}
+    # Every named SpGEMM workload (BASELINE's five configurations), on a single GPU.
+    per_config = None
+    if args.per_config and not ew and not args.rows and world == 1:
+        per_config = {}
+        for name in WORKLOAD_ORDER:
+            if name == args.workload:
+                e = head
+            else:
+                A2, B2 = workload(name)
+                e = measure(args, name, A2, B2, args.steps, args.warmup, args.e2e_steps, args.per_config_cpu_s,
+                            world, rank, local, pg, min_region_s=args.per_config_s)
+                del A2, B2
+            if rank == 0:
+                per_config[name] = {k: e[k] for k in ("value", "unit", "ms_per_step", "steps", "dtype", "products",
+                                                      "nnz_c", "effective_hbm_gbs", "frac_of_8tbs", "phases_ms",
+                                                      "roofline", "gpu_launches", "clocks", "e2e", "cpu_baseline")}
+    if rank != 0:
+        return
+    line = {
+        "metric": EWISE_METRIC if ew else METRIC,
+        "value": head["value"],
+        "unit": head["unit"],
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": head["ms_per_step"],
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": head["dtype"],
+        "data": "synthetic",
+        "config": {
+            "workload": head["workload"], "description": head["description"],
+            "m": head["m"], "k": head["k"], "n": head["n"], "nnz_a": head["nnz_a"], "nnz_b": head["nnz_b"],
+            "nnz_c": head["nnz_c"], **({"op": args.op} if ew else {"products": head["products"]}),
+            "l2": "flushed between timed steps (write of a buffer > L2)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        },
+        "effective_hbm_gbs": head["effective_hbm_gbs"],
+        "frac_of_8tbs": head["frac_of_8tbs"],
+        "phases_ms": head["phases_ms"],
+        "roofline": head["roofline"],
+        "gpu_launches": head["gpu_launches"],
+        "plan": head["plan"],
+        "clocks": head["clocks"],
+        "e2e": head["e2e"],
+        "cpu_baseline": head["cpu_baseline"],
+    }
+    if sustained is not None:
+        line["sustained"] = sustained
+    if per_config is not None:
+        line["per_config"] = per_config
     print(json.dumps(line), flush=True)
 
 
@@ -686,9 +801,16 @@ def main(argv=None) -> int:
     ap.add_argument("--ref-step-s", type=float, default=2.0, help="seconds per reference-arm step")
     ap.add_argument("--rows", type=int, default=0,
                     help="use only the first ROWS rows of A (a smaller case of the same workload, for profiling)")
-    ap.add_argument("--traffic", type=float, default=None,
-                    help="ncu DRAM bytes per numeric launch, when captured for the current kernels")
+    ap.add_argument("--per-config", dest="per_config", action="store_true", default=None,
+                    help="also measure every named SpGEMM workload (default: on without --workload)")
+    ap.add_argument("--no-per-config", dest="per_config", action="store_false")
+    ap.add_argument("--per-config-s", type=float, default=0.5, help="least seconds of timed steps per workload")
+    ap.add_argument("--per-config-cpu-s", type=float, default=3.0, help="seconds of CPU oracle work per workload")
+    ap.add_argument("--sustained-s", type=float, default=1.0,
+                    help="least seconds of the headline's second timed region (0 = skip)")
     args = ap.parse_args(argv)
+    if args.per_config is None:
+        args.per_config = args.workload == DEFAULT_WORKLOAD and "--workload" not in (argv or sys.argv[1:])
     world, rank, local, pg = dist_setup()
     try:
         if args.workload in SPMSPV_WORKLOADS:

@@ -80,3 +80,28 @@ def test_max_over_ranks_gloo():
         p.join(timeout=60)
         assert p.exitcode == 0
     assert out == {0: 3.0, 1: 3.0}
+
+
+def test_traffic_records_follow_the_kernel_source(tmp_path, monkeypatch):
+    """roofline.traffic comes from a `traffic-record:` line of a profile
+    summary, scaled from the captured rows to the full workload, and is None
+    once the kernel source no longer matches the recorded digest."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    src = tmp_path / "kern.cu"
+    src.write_text("// kernel v1\n")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "PROFILES", str(prof))
+    digest = bench.source_digest("kern.cu")
+    assert digest is not None and len(digest) == 16
+    (prof / "k.md").write_text(
+        "# capture\n\ntraffic-record: workload=w kernel=k_kernel rows=100 of=400 dram_bytes=2.5e6 "
+        f"source=kern.cu sha256={digest}\n")
+    assert bench.recorded_traffic("w", "k_kernel") == 1e7
+    assert bench.recorded_traffic("w", "other_kernel") is None
+    assert bench.recorded_traffic("other", "k_kernel") is None
+    src.write_text("// kernel v2\n")  # the kernel changed after the capture
+    assert bench.recorded_traffic("w", "k_kernel") is None
