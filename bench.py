@@ -526,8 +526,9 @@ def run_outer(args, world, rank, local, pg, A, B, dA, dB, ub, flush, stream, dev
         "effective_hbm_gbs": round(algo * args.steps * world / total_s / 1e9, 1),
         "phases_ms": {"step_min": round(min(step_ms), 4), "step_median": round(statistics.median(step_ms), 4)},
         "roofline": dict(roofline_obj(algo, statistics.mean(step_ms) / 1e3, peaks, None),
-                         kernel=f"whole outer-product SpGEMM ({args.parts} k blocks: submatrices, partial products, "
-                                "pairwise sparse additions; read-backs included)"),
+                         kernel=f"whole outer-product SpGEMM ({args.parts} k blocks inside the library: "
+                                "column-block extraction, partial products, pairwise sparse additions; "
+                                "read-backs included)"),
         "gpu_launches": int(stats.get("launches", 0)),
         "clocks": clk, "e2e": None, "cpu_baseline": None,
     }

@@ -140,6 +140,32 @@ ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_
 ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
                               ws_stream_t stream);
 
+/*
+ * ws_spgemm_outer_symbolic / ws_spgemm_outer_numeric -- C = A * B as the
+ * outer-product SpGEMM (Sec. 5.1, Fig. "SpGEMM implemented in WingSpan",
+ * outer product, with the merge level and its coalesce step of Sec. 4): the
+ * k range is split into `parts` contiguous blocks K_p; block p contributes the
+ * partial product A[:, K_p] * B[K_p, :] (a worker's own copy of C) and the
+ * copies are coalesced by pairwise sparse additions.  C's structure equals
+ * the row-wise product's (a sum of exactly 0.0 is kept); values agree up to
+ * summation order (sums per block, then block sums).
+ *   parts  >= 1 (clamped to the number of columns of A; 1 is the row-wise
+ *          product itself), else WS_ERR_INVALID_ARG
+ * Same two-pass contract as ws_spgemm_symbolic / ws_spgemm_numeric: the
+ * symbolic call writes C.rowptr, returns nnz(C) and synchronises `stream`;
+ * it computes every block's partial product and every merge except the value
+ * pass of the last one, in library-owned scratch allocated stream-ordered on
+ * `stream` (B's row blocks are views of B, A's column blocks share one buffer
+ * of nnz(A) entries).  The numeric call (asynchronous) writes C's column
+ * indices and values and releases that scratch stream-ordered.  A and B must
+ * stay unchanged in between.  Errors as for the row-wise calls; a device-side
+ * failure in any step gives WS_ERR_DEVICE.
+ */
+ws_status_t ws_spgemm_outer_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int parts, int64_t* nnz_out,
+                                     ws_stream_t stream);
+ws_status_t ws_spgemm_outer_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                                    ws_stream_t stream);
+
 /* Elementwise operations (Sec. 5.2, "Sparse Linear Algebra": C = A op B). */
 typedef enum {
   WS_EWISE_ADD = 1, /* SpAdd: C = A + B on the union of the two patterns            */

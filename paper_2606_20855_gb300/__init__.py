@@ -8,7 +8,7 @@ same function names; ``spgemm`` holds the PyTorch-facing wrapper.  Importing
 this package loads nothing; the library is loaded on first use.
 """
 
-__all__ = ["DeviceCSR", "SpGEMM", "spgemm", "spgemm_outer", "submatrix", "Ewise", "ewise", "SpMSpV", "spmspv"]
+__all__ = ["DeviceCSR", "SpGEMM", "SpGEMMOuter", "spgemm", "spgemm_outer", "submatrix", "Ewise", "ewise", "SpMSpV", "spmspv"]
 
 
 def __getattr__(name):

@@ -48,6 +48,8 @@ SIGNATURES = [
     ("ws_spmspv", _i32, [_p, _i64, _p, _p, _p, _p, ctypes.POINTER(_i64), _p]),
     ("ws_csr_submatrix_symbolic", _i32, [_p, _i64, _i64, _i64, _i64, _p, ctypes.POINTER(_i64), _p]),
     ("ws_csr_submatrix_numeric", _i32, [_p, _p, _p, _p, _p]),
+    ("ws_spgemm_outer_symbolic", _i32, [_p, _p, _p, _i32, ctypes.POINTER(_i64), _p]),
+    ("ws_spgemm_outer_numeric", _i32, [_p, _p, _p, _p, _p, _p]),
 ]
 
 EWISE_OPS = {"add": 1, "mul": 2}  # ws_ewise_op_t
@@ -107,6 +109,18 @@ def ws_spgemm_symbolic(A: int, B: int, C: int, stream: int) -> int:
 def ws_spgemm_numeric(A: int, B: int, C: int, c_colidx: int, c_vals: int, stream: int) -> None:
     _check("ws_spgemm_numeric", load().ws_spgemm_numeric(A, B, C, c_colidx or None, c_vals or None,
                                                          stream or None))
+
+
+def ws_spgemm_outer_symbolic(A: int, B: int, C: int, parts: int, stream: int) -> int:
+    nnz = ctypes.c_int64(-1)
+    _check("ws_spgemm_outer_symbolic", load().ws_spgemm_outer_symbolic(A, B, C, int(parts), ctypes.byref(nnz),
+                                                                       stream or None))
+    return nnz.value
+
+
+def ws_spgemm_outer_numeric(A: int, B: int, C: int, c_colidx: int, c_vals: int, stream: int) -> None:
+    _check("ws_spgemm_outer_numeric", load().ws_spgemm_outer_numeric(A, B, C, c_colidx or None, c_vals or None,
+                                                                     stream or None))
 
 
 def ws_ewise_symbolic(A: int, B: int, C: int, op, stream: int) -> int:

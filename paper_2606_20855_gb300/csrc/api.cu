@@ -192,6 +192,7 @@ struct Plan {
   int dense_width = 0;
   int run_limit = 64;
   int sym_launches = 0, num_launches = 0;
+  struct OuterState* outer = nullptr;  // outer-product SpGEMM between its two passes
 };
 
 }  // namespace
@@ -726,6 +727,265 @@ ws_status_t check_handle(const ws_csr_s* h, const char* name) {
   return WS_OK;
 }
 
+// ------------------------------------------------------ outer-product SpGEMM
+//
+// C = A*B with the k loop split over P workers (Sec. 5.1, Fig. "SpGEMM
+// implemented in WingSpan", outer product): worker p multiplies the column
+// block A[:, K_p] by the row block B[K_p, :] into its own copy of C, and a
+// merge level coalesces the copies (Sec. 4, coalesce).  On one GPU every
+// block's product already fills the device, so the blocks run one after
+// another on the caller's stream:
+//   - B[K_p, :] is a view of B's rows (no copy);
+//   - A[:, K_p] is extracted (count, scan, copy) into one library buffer of
+//     nnz(A) entries that every block reuses, so its size needs no read-back;
+//   - the partial product is the row-wise product of the two blocks;
+//   - the partial products are merged pairwise by sparse additions (a sum of
+//     exactly 0.0 is kept, so C's structure equals the row-wise product's).
+// The symbolic call runs everything but the value pass of the last merge,
+// whose structure pass writes C.rowptr; the numeric call runs that value pass.
+
+// A CSR matrix whose arrays the library owns (stream-ordered allocations).
+struct Owned {
+  ws_csr_s h;
+  void* rp_mem = nullptr;  // row pointer
+  void* cv_mem = nullptr;  // column indices and values
+};
+
+struct OuterState {
+  int parts = 1;
+  const ws_csr_s* A = nullptr;
+  const ws_csr_s* B = nullptr;
+  int64_t a_nnz = 0, b_nnz = 0;
+  Owned* x = nullptr;  // operands of the last merge (parts >= 2)
+  Owned* y = nullptr;
+};
+
+// Frees a plan's scratch stream-ordered on s (no device synchronisation).
+void release_plan_async(Plan* pl, cudaStream_t s);
+
+void release_owned(Owned* o, cudaStream_t s) {
+  if (!o) return;
+  release_plan_async(o->h.plan, s);
+  o->h.plan = nullptr;
+  if (o->rp_mem) cudaFreeAsync(o->rp_mem, s);
+  if (o->cv_mem) cudaFreeAsync(o->cv_mem, s);
+  delete o;
+}
+
+void release_outer(Plan* pl, cudaStream_t s) {
+  if (!pl || !pl->outer) return;
+  release_owned(pl->outer->x, s);
+  release_owned(pl->outer->y, s);
+  delete pl->outer;
+  pl->outer = nullptr;
+}
+
+void release_plan_async(Plan* pl, cudaStream_t s) {
+  if (!pl) return;
+  release_outer(pl, s);
+  DevBuf* bufs[] = {&pl->rows, &pl->slices, &pl->ranks, &pl->ew, &pl->sv, &pl->rcd, &pl->rcdb};
+  for (DevBuf* b : bufs) {
+    if (b->ptr) cudaFreeAsync(b->ptr, s);
+    b->ptr = nullptr;
+    b->bytes = 0;
+  }
+  release_host_sum(pl->host_sum);
+  delete pl;
+}
+
+// An owned m x n matrix with its row pointer allocated; entries come later.
+ws_status_t new_owned(int64_t m, int64_t n, ws_dtype_t dt, int dev, cudaStream_t s, Owned** out) {
+  *out = nullptr;
+  Owned* o = new (std::nothrow) Owned;
+  if (!o) return fail(WS_ERR_ALLOC, "host allocation failed");
+  o->h.nrows = m;
+  o->h.ncols = n;
+  o->h.nnz = 0;
+  o->h.dtype = dt;
+  o->h.device = dev;
+  const cudaError_t e = cudaMallocAsync(&o->rp_mem, 8 * static_cast<size_t>(m + 1), s);
+  if (e != cudaSuccess) {
+    delete o;
+    return fail(WS_ERR_ALLOC, "cudaMallocAsync(row pointer): %s", cudaGetErrorString(e));
+  }
+  o->h.rowptr = static_cast<int64_t*>(o->rp_mem);
+  ws_status_t st = ensure_plan(&o->h);
+  if (st != WS_OK) {
+    release_owned(o, s);
+    return st;
+  }
+  *out = o;
+  return WS_OK;
+}
+
+// Room for cap entries (column indices and values) of an owned matrix.
+ws_status_t owned_entries(Owned* o, int64_t cap, cudaStream_t s) {
+  const size_t vs = o->h.dtype == WS_F64 ? 8 : 4;
+  const size_t o_val = align_up(4 * static_cast<size_t>(cap > 0 ? cap : 1), 256);
+  const cudaError_t e = cudaMallocAsync(&o->cv_mem, o_val + vs * static_cast<size_t>(cap > 0 ? cap : 1), s);
+  if (e != cudaSuccess) return fail(WS_ERR_ALLOC, "cudaMallocAsync(%lld entries): %s", (long long)cap, cudaGetErrorString(e));
+  o->h.colidx = static_cast<int32_t*>(o->cv_mem);
+  o->h.vals = static_cast<char*>(o->cv_mem) + o_val;
+  return WS_OK;
+}
+
+// Device status word of a plan whose queued work has completed.
+ws_status_t plan_status(const Plan* pl) {
+  int st = 0;
+  WS_CUDA(cudaMemcpy(&st, &pl->dsum->status, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(status)");
+  if (st != 0) return fail(WS_ERR_DEVICE, "device status 0x%x in an outer-product step", st);
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t outer_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, int parts, cudaStream_t s,
+                                int64_t* nnz_out) {
+  Plan* pl = C->plan;
+  release_outer(pl, s);
+  const int64_t m = A->nrows, K = A->ncols, n = B->ncols;
+  const int P = static_cast<int>(parts < 1 ? 1 : (parts > K ? (K > 0 ? K : 1) : parts));
+  OuterState* os = new (std::nothrow) OuterState;
+  if (!os) return fail(WS_ERR_ALLOC, "host allocation failed");
+  os->parts = P;
+  os->A = A;
+  os->B = B;
+  os->a_nnz = A->nnz;
+  os->b_nnz = B->nnz;
+  if (P == 1) {  // one block: the row-wise product itself
+    ws_status_t st = symbolic_impl<T>(A, B, C, pl, s, nnz_out);
+    if (st != WS_OK) {
+      delete os;
+      return st;
+    }
+    pl->outer = os;
+    return WS_OK;
+  }
+  const int sms = num_sms_of(C->device);
+  int launches = 0;
+  std::vector<Owned*> partial;
+  Owned* ab = nullptr;  // the current column block of A
+  void* ex_mem = nullptr;  // the extraction's summary and scan partials
+  ws_status_t st = WS_OK;
+  auto cleanup = [&]() {
+    for (Owned* o : partial) release_owned(o, s);
+    release_owned(ab, s);
+    if (ex_mem) cudaFreeAsync(ex_mem, s);
+    delete os;
+  };
+  const size_t o_part = align_up(sizeof(DevSummary), 256);
+  cudaError_t e = cudaMallocAsync(&ex_mem, o_part + 8 * static_cast<size_t>(scan_partials_needed(m) + 1), s);
+  if (e != cudaSuccess) {
+    ex_mem = nullptr;
+    cleanup();
+    return fail(WS_ERR_ALLOC, "cudaMallocAsync(extraction scratch): %s", cudaGetErrorString(e));
+  }
+  DevSummary* ex_sum = static_cast<DevSummary*>(ex_mem);
+  int64_t* ex_part = reinterpret_cast<int64_t*>(static_cast<char*>(ex_mem) + o_part);
+  if (cudaMemsetAsync(ex_sum, 0, sizeof(DevSummary), s) != cudaSuccess ||
+      (st = new_owned(m, 1, A->dtype, C->device, s, &ab)) != WS_OK || (st = owned_entries(ab, A->nnz, s)) != WS_OK) {
+    cleanup();
+    return st != WS_OK ? st : fail(WS_ERR_CUDA, "cudaMemsetAsync(extraction summary)");
+  }
+  ab->h.nnz = A->nnz;  // capacity: the block's own count stays on the device
+  for (int p = 0; p < P && st == WS_OK; ++p) {
+    const int64_t k0 = K * p / P, k1 = K * (p + 1) / P;
+    // A[:, k0:k1], columns shifted by -k0
+    ab->h.ncols = k1 - k0;
+    if (cudaMemsetAsync(ab->h.rowptr, 0, sizeof(int64_t), s) != cudaSuccess) {
+      st = fail(WS_ERR_CUDA, "cudaMemsetAsync(block row pointer)");
+      break;
+    }
+    if (m > 0) {
+      launch_submatrix_count(A->rowptr, A->colidx, 0, m, k0, k1, ab->h.rowptr, sms, s, &launches);
+      launch_scan(ab->h.rowptr, m, ex_part, ex_sum, s, &launches);
+      launch_submatrix_copy<T>(A->rowptr, A->colidx, static_cast<const T*>(A->vals), 0, m, k0, ab->h.rowptr,
+                               ab->h.colidx, static_cast<T*>(ab->h.vals), ex_sum, sms, s, &launches);
+    }
+    // B[k0:k1, :]: a view of B's rows (positions stay absolute in B's arrays)
+    ws_csr_s bp = *B;
+    bp.plan = nullptr;
+    bp.nrows = k1 - k0;
+    bp.rowptr = B->rowptr + k0;
+    bp.nnz = K > 0 ? B->nnz * (k1 - k0) / K : 0;  // estimate: only the lane-group choice reads it
+    // the worker's partial product
+    Owned* cp = nullptr;
+    if ((st = new_owned(m, n, A->dtype, C->device, s, &cp)) != WS_OK) break;
+    partial.push_back(cp);
+    int64_t nnz_p = 0;
+    if ((st = symbolic_impl<T>(&ab->h, &bp, &cp->h, cp->h.plan, s, &nnz_p)) != WS_OK) break;
+    cp->h.nnz = nnz_p;
+    if ((st = owned_entries(cp, nnz_p, s)) != WS_OK) break;
+    if ((st = numeric_impl<T>(&ab->h, &bp, &cp->h, cp->h.plan, s)) != WS_OK) break;
+    launches += cp->h.plan->sym_launches + cp->h.plan->num_launches;
+  }
+  if (st == WS_OK) {  // every extraction has completed (each block's structure pass synchronised)
+    int ex_status = 0;
+    if (cudaMemcpy(&ex_status, &ex_sum->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+      st = fail(WS_ERR_CUDA, "cudaMemcpy(extraction status)");
+    else if (ex_status != 0)
+      st = fail(WS_ERR_DEVICE, "device status 0x%x in a column-block extraction", ex_status);
+  }
+  release_owned(ab, s);
+  ab = nullptr;
+  // merge levels: pairwise sparse additions until two copies are left
+  while (st == WS_OK && partial.size() > 2) {
+    std::vector<Owned*> next;
+    size_t i = 0;
+    for (; i + 1 < partial.size() && st == WS_OK; i += 2) {
+      Owned* x = partial[i];
+      Owned* y = partial[i + 1];
+      Owned* z = nullptr;
+      if ((st = new_owned(m, n, A->dtype, C->device, s, &z)) != WS_OK) break;
+      next.push_back(z);
+      int64_t nz = 0;
+      if ((st = ewise_symbolic_impl<T>(&x->h, &y->h, &z->h, z->h.plan, kEwiseAdd, s, &nz)) != WS_OK) break;
+      if ((st = plan_status(x->h.plan)) != WS_OK || (st = plan_status(y->h.plan)) != WS_OK) break;
+      z->h.nnz = nz;
+      if ((st = owned_entries(z, nz, s)) != WS_OK) break;
+      if (nz > 0) launch_ewise_numeric<T>(make_ewise<T>(&x->h, &y->h, &z->h, z->h.plan), sms, s, &launches);
+      launches += z->h.plan->sym_launches;
+      release_owned(x, s);  // stream-ordered: the value pass above still reads them
+      release_owned(y, s);
+      partial[i] = partial[i + 1] = nullptr;
+    }
+    for (; i < partial.size(); ++i) {
+      if (partial[i]) next.push_back(partial[i]);
+      partial[i] = nullptr;
+    }
+    for (Owned* o : partial) release_owned(o, s);
+    partial.swap(next);
+  }
+  if (st == WS_OK) {  // the last merge's structure pass writes C.rowptr
+    st = ewise_symbolic_impl<T>(&partial[0]->h, &partial[1]->h, C, pl, kEwiseAdd, s, nnz_out);
+    if (st == WS_OK && (st = plan_status(partial[0]->h.plan)) == WS_OK) st = plan_status(partial[1]->h.plan);
+  }
+  cudaFreeAsync(ex_mem, s);
+  ex_mem = nullptr;
+  if (st != WS_OK) {
+    cleanup();
+    return st;
+  }
+  os->x = partial[0];
+  os->y = partial[1];
+  partial.clear();
+  pl->outer = os;
+  pl->sym_launches += launches;
+  return WS_OK;
+}
+
+template <typename T>
+ws_status_t outer_numeric_impl(ws_csr_s* C, cudaStream_t s) {
+  Plan* pl = C->plan;
+  OuterState* os = pl->outer;
+  if (os->parts == 1) return numeric_impl<T>(os->A, os->B, C, pl, s);
+  pl->num_launches = 0;
+  if (C->nnz > 0)
+    launch_ewise_numeric<T>(make_ewise<T>(&os->x->h, &os->y->h, C, pl), num_sms_of(C->device), s, &pl->num_launches);
+  WS_CUDA(cudaGetLastError(), "outer-product merge launch");
+  release_outer(pl, s);  // stream-ordered: the copies stay valid for the pass just queued
+  return WS_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -799,6 +1059,7 @@ ws_status_t ws_spgemm_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int64_t* nnz_
   if ((st = prepare_output(A, B, C)) != WS_OK) return st;
   Plan* pl = C->plan;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  release_outer(pl, s);
   C->nnz = -1;
   if (A->dtype == WS_F64) return symbolic_impl<double>(A, B, C, pl, s, nnz_out);
   return symbolic_impl<float>(A, B, C, pl, s, nnz_out);
@@ -824,6 +1085,52 @@ ws_status_t ws_spgemm_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_col
   return numeric_impl<float>(A, B, C, pl, s);
 }
 
+ws_status_t ws_spgemm_outer_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int parts, int64_t* nnz_out,
+                                     ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  if (!nnz_out) return fail(WS_ERR_INVALID_ARG, "nnz_out is NULL");
+  if (parts < 1) return fail(WS_ERR_INVALID_ARG, "parts must be at least 1, got %d", parts);
+  if (C == A || C == B) return fail(WS_ERR_INVALID_ARG, "C must be a separate output handle");
+  if (A->ncols != B->nrows)
+    return fail(WS_ERR_SHAPE, "A is %lldx%lld but B is %lldx%lld", (long long)A->nrows, (long long)A->ncols,
+                (long long)B->nrows, (long long)B->ncols);
+  if (C->nrows != A->nrows || C->ncols != B->ncols)
+    return fail(WS_ERR_SHAPE, "C is %lldx%lld, expected %lldx%lld", (long long)C->nrows, (long long)C->ncols,
+                (long long)A->nrows, (long long)B->ncols);
+  if (A->dtype != B->dtype || C->dtype != A->dtype) return fail(WS_ERR_DTYPE, "A, B and C dtypes differ");
+  if (A->nnz > 0 && B->nrows == 0) return fail(WS_ERR_INVALID_CSR, "A has entries but B has no rows");
+  if ((st = prepare_output(A, B, C)) != WS_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  C->nnz = -1;
+  if (A->dtype == WS_F64) return outer_symbolic_impl<double>(A, B, C, parts, s, nnz_out);
+  return outer_symbolic_impl<float>(A, B, C, parts, s, nnz_out);
+}
+
+ws_status_t ws_spgemm_outer_numeric(ws_csr_t A, ws_csr_t B, ws_csr_t C, int32_t* c_colidx, void* c_vals,
+                                    ws_stream_t stream) {
+  g_last_error.clear();
+  ws_status_t st;
+  if ((st = check_handle(A, "A")) != WS_OK || (st = check_handle(B, "B")) != WS_OK ||
+      (st = check_handle(C, "C")) != WS_OK)
+    return st;
+  Plan* pl = C->plan;
+  if (!pl || !pl->ready || !pl->outer)
+    return fail(WS_ERR_STATE, "numeric called before a successful outer-product symbolic pass");
+  const OuterState* os = pl->outer;
+  if (os->A != A || os->B != B || os->a_nnz != A->nnz || os->b_nnz != B->nnz)
+    return fail(WS_ERR_STATE, "numeric called with other operands than the symbolic pass");
+  if (C->nnz > 0 && (!c_colidx || !c_vals)) return fail(WS_ERR_INVALID_ARG, "c_colidx/c_vals NULL with nnz(C) > 0");
+  C->colidx = c_colidx;
+  C->vals = c_vals;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (A->dtype == WS_F64) return outer_numeric_impl<double>(C, s);
+  return outer_numeric_impl<float>(C, s);
+}
+
 ws_status_t ws_ewise_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int op, int64_t* nnz_out, ws_stream_t stream) {
   g_last_error.clear();
   ws_status_t st;
@@ -840,6 +1147,7 @@ ws_status_t ws_ewise_symbolic(ws_csr_t A, ws_csr_t B, ws_csr_t C, int op, int64_
                 (long long)A->nrows, (long long)A->ncols);
   if ((st = prepare_output(A, B, C)) != WS_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  release_outer(C->plan, s);
   C->nnz = -1;
   const int kop = op == WS_EWISE_ADD ? kEwiseAdd : kEwiseMul;
   if (A->dtype == WS_F64) return ewise_symbolic_impl<double>(A, B, C, C->plan, kop, s, nnz_out);
@@ -989,8 +1297,9 @@ ws_status_t ws_csr_destroy(ws_csr_t h) {
   if (!h) return WS_OK;
   if (h->plan) {
     if (h->plan->rows.ptr || h->plan->slices.ptr || h->plan->ranks.ptr || h->plan->ew.ptr || h->plan->sv.ptr ||
-        h->plan->rcd.ptr || h->plan->rcdb.ptr)
+        h->plan->rcd.ptr || h->plan->rcdb.ptr || h->plan->outer)
       cudaDeviceSynchronize();
+    release_outer(h->plan, nullptr);
     h->plan->rows.release();
     h->plan->slices.release();
     h->plan->ranks.release();

@@ -269,8 +269,39 @@ def submatrix(A: DeviceCSR, r0: int, r1: int, c0: int, c1: int, stream=None, sta
                 _abi.ws_csr_destroy(h)
 
 
-def _run(op, stats: dict | None, stream=None) -> DeviceCSR:
-    with op:
+class SpGEMMOuter(SpGEMM):
+    """A reusable outer-product product C = A*B (ws_spgemm_outer_symbolic /
+    ws_spgemm_outer_numeric): the k range is split into `parts` blocks, each
+    block's partial product is a worker's own copy of C and the copies are
+    coalesced by sparse additions, all inside the library.  Same interface as
+    :class:`SpGEMM`."""
+
+    def __init__(self, A: DeviceCSR, B: DeviceCSR, parts: int = 4, validate: bool = False, stream=None):
+        super().__init__(A, B, validate=validate, stream=stream)
+        self.parts = int(parts)
+
+    def symbolic(self, stream=None) -> int:
+        self.nnz = _abi.ws_spgemm_outer_symbolic(self._hA, self._hB, self._hC, self.parts, _stream_handle(stream))
+        return self.nnz
+
+    def numeric(self, out: DeviceCSR | None = None, stream=None) -> DeviceCSR:
+        if self.nnz is None:
+            raise RuntimeError("symbolic() must run before numeric()")
+        if out is None or out.nnz != self.nnz:
+            colidx = torch.empty(self.nnz, dtype=torch.int32, device=self.device)
+            vals = torch.empty(self.nnz, dtype=self.A.dtype, device=self.device)
+            out = DeviceCSR(self.A.nrows, self.B.ncols, self.c_rowptr, colidx, vals)
+        _abi.ws_spgemm_outer_numeric(self._hA, self._hB, self._hC, out.colidx.data_ptr() if self.nnz else 0,
+                                     out.vals.data_ptr() if self.nnz else 0, _stream_handle(stream))
+        return out
+
+
+def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None, stats: dict | None = None) -> DeviceCSR:
+    """C = A*B as the outer-product SpGEMM of Sec. 5.1 (see :class:`SpGEMMOuter`).
+    `stats["launches"]`, when given, is increased by the kernel launches queued."""
+    if A.ncols != B.nrows:
+        raise ValueError(f"shape mismatch: A is {A.nrows}x{A.ncols}, B is {B.nrows}x{B.ncols}")
+    with SpGEMMOuter(A, B, parts, stream=stream) as op:
         op.symbolic(stream)
         C = op.numeric(stream=stream)
         op.wait(stream)
@@ -278,32 +309,6 @@ def _run(op, stats: dict | None, stream=None) -> DeviceCSR:
             info = op.plan_info()
             stats["launches"] = stats.get("launches", 0) + info["symbolic_launches"] + info["numeric_launches"]
     return C
-
-
-def spgemm_outer(A: DeviceCSR, B: DeviceCSR, parts: int = 4, stream=None, stats: dict | None = None) -> DeviceCSR:
-    """C = A*B as the outer-product SpGEMM of Sec. 5.1: the k range is split
-    into `parts` contiguous blocks, block p contributes the partial product
-    A[:, K_p] * B[K_p, :] (a worker's own copy of C, computed by the row-wise
-    kernels), and the partial products are coalesced by pairwise sparse
-    additions (the merge level).  Same structure as spgemm(); values equal
-    up to summation order.  `stats["launches"]` counts the kernel launches."""
-    if A.ncols != B.nrows:
-        raise ValueError(f"shape mismatch: A is {A.nrows}x{A.ncols}, B is {B.nrows}x{B.ncols}")
-    K = A.ncols
-    parts = max(1, min(int(parts), max(K, 1)))
-    bounds = [(K * p // parts, K * (p + 1) // parts) for p in range(parts)]
-    partial = []
-    for k0, k1 in bounds:
-        Ap = submatrix(A, 0, A.nrows, k0, k1, stream, stats)
-        Bp = submatrix(B, k0, k1, 0, B.ncols, stream, stats)
-        partial.append(_run(SpGEMM(Ap, Bp, stream=stream), stats, stream))
-    while len(partial) > 1:
-        merged = [_run(Ewise(partial[i], partial[i + 1], "add", stream=stream), stats, stream)
-                  for i in range(0, len(partial) - 1, 2)]
-        if len(partial) % 2:
-            merged.append(partial[-1])
-        partial = merged
-    return partial[0]
 
 
 def spgemm(A: DeviceCSR, B: DeviceCSR, validate: bool = False, stream=None) -> DeviceCSR:

@@ -101,3 +101,28 @@ def test_outer_cancellation_and_empty():
     W = random_csr(5, 6, 0.5, np.random.default_rng(2), np.float64, "sym")
     rowptr, colidx, vals = _outer(Z, W, 3)
     assert rowptr.tolist() == [0, 0, 0, 0] and colidx.size == 0
+
+
+def test_outer_repeated_on_one_handle_and_errors():
+    """The same operator run twice gives the same product; the ABI refuses
+    parts < 1 and a numeric pass before the symbolic pass."""
+    from paper_2606_20855_gb300.spgemm import SpGEMMOuter
+    rng = np.random.default_rng(9)
+    A = random_csr(150, 90, 0.06, rng, np.float64, "sym")
+    B = random_csr(90, 120, 0.08, rng, np.float64, "sym")
+    dA, dB = DeviceCSR.from_host(A, DEV), DeviceCSR.from_host(B, DEV)
+    with SpGEMMOuter(dA, dB, parts=3) as op:
+        with pytest.raises(_abi.WsError, match="WS_ERR_STATE"):
+            _abi.ws_spgemm_outer_numeric(op._hA, op._hB, op._hC, 0, 0, 0)
+        results = []
+        for _ in range(2):
+            op.symbolic()
+            C = op.numeric()
+            op.wait()
+            results.append(C.to_host())
+        for rowptr, colidx, vals in results:
+            assert_matches_oracle(A, B, rowptr, colidx, vals)
+        assert np.array_equal(results[0][1], results[1][1])
+        op.parts = 0
+        with pytest.raises(_abi.WsError, match="WS_ERR_INVALID_ARG"):
+            op.symbolic()
