@@ -599,8 +599,25 @@ def e2e_measure(A, B, make_op, same, device, steps, world, pg, nnz, algo_bytes, 
     h2d = sum(t.numel() * t.element_size() for t in hA) + (0 if same else sum(t.numel() * t.element_size() for t in hB))
     d2h = h_rp.numel() * 8 + h_col.numel() * 4 + h_val.numel() * h_val.element_size()
     work = algo_bytes if ew else 2.0 * float(products)
+    # The host link alone: the device-to-host copy of C's arrays from a device
+    # buffer to the same pinned buffers (copy engines), timed by itself.
+    dcol = torch.empty(max(nnz, 1), dtype=torch.int32, device=device)
+    dval = torch.empty(max(nnz, 1), dtype=h_val.dtype, device=device)
+    torch.cuda.synchronize(device)
+    t0 = time.perf_counter()
+    h_col.copy_(dcol[:nnz], non_blocking=True)
+    h_val.copy_(dval[:nnz], non_blocking=True)
+    torch.cuda.synchronize(device)
+    copy_s = time.perf_counter() - t0
+    del dcol, dval
+    link_gbs = (h_col.numel() * 4 + h_val.numel() * h_val.element_size()) / max(copy_s, 1e-9) / 1e9
     return {"value": round(work * steps * world / e2e_s / 1e9, 3), "unit": "GB/s" if ew else "GFLOP/s",
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "ms_per_step": round(1e3 * e2e_s / steps, 3),
+            "host_link": {"d2h_gbs": round(link_gbs, 1),
+                          "c_copy_ms": round(1e3 * copy_s, 3),
+                          "c_copy_share_of_step": round(copy_s / (e2e_s / steps), 3),
+                          "note": "device-to-host copy of C's arrays alone, pinned host memory"}}
 
 
 def measure(args, name, A, B, steps, warmup, e2e_steps, cpu_s, world, rank, local, pg, min_region_s=0.0,
