@@ -190,7 +190,7 @@ TUNING_KEYS = {"hash_max_products": 1, "run_limit": 2, "dense_width": 3, "bitmap
                "dense_rows_max_a": 6, "wide_bitmap_span": 7, "ewise_lanes": 8, "ewise_chunk": 9}
 TUNING_DEFAULTS = {"hash_max_products": 4096, "run_limit": 64, "dense_width": 0, "bitmap_span": 65536,
                    "register_rows_max_a": 16, "dense_rows_max_a": 8192, "wide_bitmap_span": 1 << 20,
-                   "ewise_lanes": 1, "ewise_chunk": 64}
+                   "ewise_lanes": -1, "ewise_chunk": 64}
 
 
 def ws_set_tuning(key, value: int) -> None:

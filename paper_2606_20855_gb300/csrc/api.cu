@@ -34,7 +34,7 @@ int g_rcd_max_a = kRcdDefaultMaxA;
 int64_t g_wb_span = kWbMaxSpan;
 int g_run_limit = 64;
 int g_dense_width = 0;  // 0 = default per value type
-int g_ewise_lanes = 1;  // elementwise: lanes per chunk (0 = from the mean row length)
+int g_ewise_lanes = -1;  // elementwise: lanes per chunk (0 = lane groups from the mean row length, -1 = automatic)
 int64_t g_ewise_diag = 64;  // elementwise, one thread per chunk: merged positions per chunk
 constexpr int kLongRowThreshold = 128;
 
@@ -605,8 +605,13 @@ ws_status_t ewise_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* 
   pl->num_launches = 0;
   pl->ew_op = op;
   const int64_t merged = A->nnz + B->nnz;
-  pl->ew_group = g_ewise_lanes > 0 ? g_ewise_lanes : ewise_group_for(m, merged);
-  pl->ew_diag = pl->ew_group == 1 ? g_ewise_diag : 16 * static_cast<int64_t>(pl->ew_group);
+  // automatic: one thread per chunk for short rows (power-law graphs), a warp
+  // per 64-position chunk once rows average a whole chunk
+  const bool long_rows = m > 0 && merged >= static_cast<int64_t>(kEwiseRankChunk) * m;
+  pl->ew_group = g_ewise_lanes > 0 ? g_ewise_lanes
+               : g_ewise_lanes == 0 ? ewise_group_for(m, merged) : (long_rows ? kEwiseRankGroup : 1);
+  pl->ew_diag = pl->ew_group == 1 ? g_ewise_diag
+              : pl->ew_group == kEwiseRankGroup ? kEwiseRankChunk : 16 * static_cast<int64_t>(pl->ew_group);
   pl->ew_nc_max = m + merged / pl->ew_diag + 1;  // row i has at most 1 + len_i / diag chunks
   ws_status_t st = carve_ewise(pl, m, pl->ew_nc_max, s);
   if (st != WS_OK) return st;
@@ -1397,8 +1402,9 @@ ws_status_t ws_set_tuning(int key, int64_t value) {
       g_wb_span = value;
       return WS_OK;
     case 8:
-      if (value != 0 && value != 1 && value != 4 && value != 8 && value != 16 && value != 32)
-        return fail(WS_ERR_INVALID_ARG, "elementwise lanes per chunk must be 0, 1, 4, 8, 16 or 32");
+      if (value != -1 && value != 0 && value != 1 && value != 4 && value != 8 && value != 16 && value != 32 &&
+          value != kEwiseRankGroup)
+        return fail(WS_ERR_INVALID_ARG, "elementwise lanes per chunk must be -1, 0, 1, 4, 8, 16, 32 or 64");
       g_ewise_lanes = static_cast<int>(value);
       return WS_OK;
     case 9:

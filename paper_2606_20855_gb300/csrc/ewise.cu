@@ -453,6 +453,205 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_kernel(cons
   if (bad) atomicOr(&p.sum->status, kErrCount);
 }
 
+// A warp per chunk, chunks taken 32 at a time (kEwiseRankChunk merged
+// positions each).  Lane l first fetches the bounds of chunk t0 + l (row, the split of
+// each list, C offset), so the dependent loads of 32 chunks overlap; then the
+// warp takes the chunks in turn.  A chunk's parts of the two lists are staged
+// in shared memory with coalesced loads (the next chunk's are loaded while the
+// current one is merged), and every entry finds its place by a binary search
+// in the other part: for A entry x, lb = #B entries below it and whether B
+// holds its column; for B entry y, the same against A.  Ballots over the
+// "has an equal partner" flags give the pairs below each entry, so
+//   SpAdd:    rank(A x) = x + lb - pairs below x          (value a + b at a pair)
+//             rank(B y) = y + lb - pairs below y, B entries with a partner skipped
+//   Hadamard: rank(A x) = pairs below x, A entries without a partner skipped
+// and the count is na + nb - pairs (SpAdd) or pairs (Hadamard).  The outputs
+// of a chunk are one contiguous run of C written in order.
+constexpr int kRankSlots = 96;  // staged entries per list (a chunk part holds at most kEwiseRankChunk + 1)
+static_assert(kEwiseRankChunk + 1 <= kRankSlots, "a chunk's part of a list fits the staging");
+constexpr int kRankWarps = kEwThreads / 32;
+
+// First position in s[0..n) holding a value >= x (n if none).
+__device__ __forceinline__ int lower_bound_smem(const int* s, int n, int x) {
+  int lo = 0, hi = n;
+#pragma unroll 1
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (s[mid] < x) {
+      lo = mid + 1;
+    } else {
+      hi = mid;
+    }
+  }
+  return lo;
+}
+
+template <typename T, int OP, bool FILL>
+__global__ void __launch_bounds__(kEwThreads) ew_rank_kernel(const EwisePlan<T> p) {
+  __shared__ int s_ac[kRankWarps][kRankSlots], s_bc[kRankWarps][kRankSlots];
+  __shared__ T s_av[kRankWarps][FILL ? kRankSlots : 1], s_bv[kRankWarps][FILL ? kRankSlots : 1];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int* ac = s_ac[w];
+  int* bc = s_bc[w];
+  T* av = s_av[w];
+  T* bv = s_bv[w];
+  const int64_t nc = p.chunk_begin[p.m];
+  const int64_t gwarp = static_cast<int64_t>(blockIdx.x) * kRankWarps + w;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kRankWarps;
+  bool bad = false;
+  for (int64_t t0 = gwarp * 32; t0 < p.nc_max; t0 += nwarps * 32) {
+    // bounds of chunk t0 + lane
+    const int64_t c = t0 + lane;
+    int64_t ga = 0, gb = 0, o0 = 0, cap = 0;
+    int na = 0, nb = 0;
+    const bool valid = c < nc;
+    if (!FILL && c >= nc && c < p.nc_max) p.chunk_off[c + 1] = 0;
+    if (valid) {
+      const int32_t row = p.chunk_row[c];
+      const int64_t k = c - p.chunk_begin[row];
+      const int64_t a0 = p.A.rowptr[row], ra = p.A.rowptr[row + 1] - a0;
+      const int64_t b0 = p.B.rowptr[row], rb = p.B.rowptr[row + 1] - b0;
+      const int32_t* a = p.A.colidx + a0;
+      const int32_t* b = p.B.colidx + b0;
+      const int64_t d0 = k * p.diag;
+      const int64_t d1 = d0 + p.diag < ra + rb ? d0 + p.diag : ra + rb;
+      int64_t i0 = 0, j0 = 0, i1 = ra, j1 = rb;
+      if constexpr (!FILL) {
+        if (d0 > 0) merge_split(a, ra, b, rb, d0, &i0, &j0);
+        if (d1 < ra + rb) merge_split(a, ra, b, rb, d1, &i1, &j1);
+        p.chunk_split[c] = 2 * i0 + (j0 - (d0 - i0));
+      } else {
+        auto decode = [&](int64_t d, int64_t code, int64_t* i, int64_t* j) {
+          const int64_t lo = d - rb > 0 ? d - rb : 0, hi = d < ra ? d : ra;
+          const int64_t x = code >> 1;
+          *i = x < lo ? lo : (x > hi ? hi : x);
+          const int64_t y = d - *i + (code & 1);
+          *j = y > rb ? rb : y;
+        };
+        decode(d0, p.chunk_split[c], &i0, &j0);
+        if (d1 < ra + rb) decode(d1, p.chunk_split[c + 1], &i1, &j1);
+        o0 = p.chunk_off[c];
+        cap = p.chunk_off[c + 1] - o0;
+      }
+      ga = a0 + i0;
+      gb = b0 + j0;
+      const int64_t la = i1 - i0 > 0 ? i1 - i0 : 0, lb = j1 - j0 > 0 ? j1 - j0 : 0;
+      if (la > kRankSlots || lb > kRankSlots) bad = true;  // cannot happen for kEwiseRankChunk-position chunks
+      na = static_cast<int>(la < kRankSlots ? la : kRankSlots);
+      nb = static_cast<int>(lb < kRankSlots ? lb : kRankSlots);
+    }
+    const unsigned vmask = __ballot_sync(kFull, valid);
+    const int nq = 32 - __clz(vmask);  // chunks of this tile in use (a prefix of the lanes)
+    // entries of chunk q held in registers: lane l takes positions l, l + 32, l + 64
+    int pac[3], pbc[3];
+    T pav[3], pbv[3];
+    auto fetch = [&](int q) {
+      const int64_t cga = __shfl_sync(kFull, ga, q), cgb = __shfl_sync(kFull, gb, q);
+      const int cna = __shfl_sync(kFull, na, q), cnb = __shfl_sync(kFull, nb, q);
+#pragma unroll
+      for (int r = 0; r < 3; ++r) {
+        const int e = lane + 32 * r;
+        pac[r] = e < cna ? p.A.colidx[cga + e] : 0;
+        pbc[r] = e < cnb ? p.B.colidx[cgb + e] : 0;
+        if constexpr (FILL) {
+          pav[r] = e < cna ? p.A.vals[cga + e] : T(0);
+          pbv[r] = e < cnb ? p.B.vals[cgb + e] : T(0);
+        }
+      }
+    };
+    if (nq > 0) fetch(0);
+    for (int q = 0; q < nq; ++q) {
+      const int cna = __shfl_sync(kFull, na, q), cnb = __shfl_sync(kFull, nb, q);
+      const int64_t co0 = __shfl_sync(kFull, o0, q), ccap = __shfl_sync(kFull, cap, q);
+#pragma unroll
+      for (int r = 0; r < 3; ++r) {
+        ac[lane + 32 * r] = pac[r];
+        bc[lane + 32 * r] = pbc[r];
+        if constexpr (FILL) {
+          av[lane + 32 * r] = pav[r];
+          bv[lane + 32 * r] = pbv[r];
+        }
+      }
+      __syncwarp();
+      if (q + 1 < nq) fetch(q + 1);  // in flight while this chunk is ranked
+      // A side: position in B and equal partner
+      int lbA[3];
+      unsigned eqA[3];
+#pragma unroll
+      for (int r = 0; r < 3; ++r) {
+        const int x = lane + 32 * r;
+        lbA[r] = 0;
+        bool eq = false;
+        if (x < cna) {
+          const int col = ac[x];
+          lbA[r] = lower_bound_smem(bc, cnb, col);
+          eq = lbA[r] < cnb && bc[lbA[r]] == col;
+        }
+        eqA[r] = __ballot_sync(kFull, eq);
+      }
+      const int pairs = __popc(eqA[0]) + __popc(eqA[1]) + __popc(eqA[2]);
+      const int count = OP == kEwiseAdd ? cna + cnb - pairs : pairs;
+      if constexpr (!FILL) {
+        if (lane == q) p.chunk_off[c + 1] = count;
+      } else {
+        if (count != ccap) bad = true;
+        const unsigned below = (1u << lane) - 1u;
+#pragma unroll
+        for (int r = 0; r < 3; ++r) {
+          const int x = lane + 32 * r;
+          if (x >= cna) continue;
+          int pb = __popc(eqA[r] & below);  // pairs below x
+          for (int r2 = 0; r2 < r; ++r2) pb += __popc(eqA[r2]);
+          const bool eq = (eqA[r] >> lane) & 1u;
+          if (OP == kEwiseAdd) {
+            const int64_t rank = x + lbA[r] - pb;
+            if (rank < ccap) {
+              p.c_colidx[co0 + rank] = ac[x];
+              p.c_vals[co0 + rank] = eq ? av[x] + bv[lbA[r]] : av[x];
+            }
+          } else if (eq) {
+            if (pb < ccap) {
+              p.c_colidx[co0 + pb] = ac[x];
+              p.c_vals[co0 + pb] = av[x] * bv[lbA[r]];
+            }
+          }
+        }
+        if constexpr (OP == kEwiseAdd) {
+          // B side: entries without a partner, placed among A
+          int lbB[3];
+          unsigned eqB[3];
+#pragma unroll
+          for (int r = 0; r < 3; ++r) {
+            const int y = lane + 32 * r;
+            lbB[r] = 0;
+            bool eq = false;
+            if (y < cnb) {
+              const int col = bc[y];
+              lbB[r] = lower_bound_smem(ac, cna, col);
+              eq = lbB[r] < cna && ac[lbB[r]] == col;
+            }
+            eqB[r] = __ballot_sync(kFull, eq);
+          }
+#pragma unroll
+          for (int r = 0; r < 3; ++r) {
+            const int y = lane + 32 * r;
+            if (y >= cnb || ((eqB[r] >> lane) & 1u)) continue;
+            int pb = __popc(eqB[r] & below);
+            for (int r2 = 0; r2 < r; ++r2) pb += __popc(eqB[r2]);
+            const int64_t rank = y + lbB[r] - pb;
+            if (rank < ccap) {
+              p.c_colidx[co0 + rank] = bc[y];
+              p.c_vals[co0 + rank] = bv[y];
+            }
+          }
+        }
+      }
+      __syncwarp();  // the staged parts are overwritten by the next chunk
+    }
+  }
+  if (bad) atomicOr(&p.sum->status, kErrCount);
+}
+
 // C.rowptr[i] = output offset of the first chunk of row i (i = 0..m; the
 // first chunk past row m - 1 is the end).
 __global__ void __launch_bounds__(kEwThreads) ew_rowptr_kernel(int64_t m, const int64_t* chunk_begin,
@@ -476,6 +675,10 @@ void launch_merge(const EwisePlan<T>& p, int num_sms, cudaStream_t s) {
 
 template <typename T, int OP, bool FILL>
 void launch_merge_g(const EwisePlan<T>& p, int num_sms, cudaStream_t s) {
+  if (p.group == kEwiseRankGroup) {
+    ew_rank_kernel<T, OP, FILL><<<grid_for((p.nc_max + 31) / 32, kRankWarps, num_sms, 8), kEwThreads, 0, s>>>(p);
+    return;
+  }
   if (p.group == 1) {
     ew_merge_seq_kernel<T, OP, FILL><<<grid_for(p.nc_max, kEwThreads, num_sms, 8), kEwThreads, 0, s>>>(p);
     return;

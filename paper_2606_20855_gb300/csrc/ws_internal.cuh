@@ -164,6 +164,8 @@ struct RowPlan {
 // Elementwise operations C = A op B on CSR matrices of one shape.
 constexpr int kEwiseAdd = 1;  // SpAdd: pattern union, values added
 constexpr int kEwiseMul = 2;  // Hadamard product: pattern intersection, values multiplied
+constexpr int kEwiseRankGroup = 64;  // EwisePlan::group of the warp-per-chunk ranking kernels
+constexpr int kEwiseRankChunk = 64;  // their merged positions per chunk
 
 template <typename T>
 struct EwisePlan {
@@ -181,7 +183,8 @@ struct EwisePlan {
   int64_t* partials;     // scan scratch for max(m, nc_max) entries
   DevSummary* sum;
   int64_t diag;          // merged positions per chunk
-  int group;             // lanes per chunk (1: one thread merges entry by entry; 4, 8, 16, 32: windows)
+  int group;             // lanes per chunk (1: one thread merges entry by entry; 4, 8, 16, 32: windows;
+                         // kEwiseRankGroup: a warp per chunk ranks every entry by binary search)
   int op;                // kEwiseAdd or kEwiseMul
 };
 template <typename T>

@@ -53,9 +53,10 @@ def check(A, B, op, validate=False):
     return info
 
 
-# lanes per chunk: 1 (one thread per chunk, the default) and 0 (lane groups
-# of 4..32 sized from the mean row length)
-LANES = [1, 0]
+# lanes per chunk: 1 (one thread per chunk), 0 (lane groups of 4..32 sized
+# from the mean row length) and 64 (a warp per 64-position chunk ranking every
+# entry by binary search)
+LANES = [1, 0, 64]
 
 
 @pytest.mark.parametrize("lanes", LANES)
@@ -103,7 +104,7 @@ def _long_rows(m, n, lens, rng, overlap):
     return build(ra), build(rb)
 
 
-@pytest.mark.parametrize("lanes,chunk", [(1, 64), (1, 2), (1, 7), (0, 64), (32, 64)])
+@pytest.mark.parametrize("lanes,chunk", [(1, 64), (1, 2), (1, 7), (0, 64), (32, 64), (64, 64), (-1, 64)])
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("overlap", [0.0, 0.5, 1.0])
 def test_long_rows_many_chunks(overlap, op, lanes, chunk):
@@ -151,18 +152,20 @@ def test_cancelled_sums_are_kept():
 
 
 @pytest.mark.slow
+@pytest.mark.parametrize("lanes", [None, 1, 64])
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("name", list(EWISE_WORKLOADS))
-def test_full_size_workloads(name, op):
+def test_full_size_workloads(name, op, lanes):
     A, B = ewise_workload(name)
     dA = DeviceCSR.from_host(A, "cuda:0")
     dB = dA if B is A else DeviceCSR.from_host(B, "cuda:0")
-    with Ewise(dA, dB, op) as e:
-        e.symbolic()
-        C = e.numeric()
-        e.wait()
-        device_invariants(C)
-        rowptr, colidx, vals = C.to_host()
+    with tuning(**({} if lanes is None else {"ewise_lanes": lanes})):
+        with Ewise(dA, dB, op) as e:
+            e.symbolic()
+            C = e.numeric()
+            e.wait()
+            device_invariants(C)
+            rowptr, colidx, vals = C.to_host()
     ref = oracle_ewise(A, B, op)
     np.testing.assert_array_equal(rowptr, ref.rowptr)
     np.testing.assert_array_equal(colidx, ref.colidx)
