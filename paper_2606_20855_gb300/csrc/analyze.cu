@@ -112,8 +112,13 @@ __device__ __forceinline__ void flush_counts(const RowPlan<T>& p, int* s_seg, lo
   }
 }
 
+// Longest row a warp analyses; longer rows take a whole CTA.
+constexpr int64_t kMidRowMax = 2048;
+
 // One thread per row for rows with at most long_threshold stored entries;
-// longer rows are queued for analyze_long_kernel.
+// longer rows are queued in long_rows for analyze_long_kernel: rows up to
+// kMidRowMax entries from the front (a warp per row), the others from the back
+// (a CTA per row).
 template <typename T>
 __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const AnalyzeParams ap,
                                                       int32_t* long_rows, const int32_t* rows) {
@@ -133,7 +138,11 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
     const int64_t i = rows ? rows[t] : t;
     const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
     if (e - s > ap.long_threshold) {
-      long_rows[atomicAdd(&p.sum->n_long, 1)] = static_cast<int32_t>(i);
+      if (e - s <= kMidRowMax) {
+        long_rows[atomicAdd(&p.sum->n_mid, 1)] = static_cast<int32_t>(i);
+      } else {
+        long_rows[ap.m - 1 - atomicAdd(&p.sum->n_long, 1)] = static_cast<int32_t>(i);
+      }
       continue;
     }
     long long ub = 0;
@@ -155,8 +164,12 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
 }
 
-// One CTA per long row (a power-law row can hold tens of thousands of
-// entries, and its three dependent loads per entry are a latency chain):
+// Rows queued by analyze_kernel.  First one CTA per long row (a power-law
+// row can hold tens of thousands of entries, and its three dependent loads
+// per entry are a latency chain), then one warp per row of long_threshold + 1
+// .. kMidRowMax entries (the lanes stride over the entries, eight in flight
+// each, and warp reductions give the product count and the column range).
+// For a long row:
 // threads stride over the row's stored entries, eight in flight each, and
 // the CTA reduces the product count and column range.
 template <typename T>
@@ -177,7 +190,7 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nlong = *reinterpret_cast<volatile int*>(&p.sum->n_long);
   for (int64_t w = blockIdx.x; w < nlong; w += gridDim.x) {
-    const int64_t i = long_rows[w];
+    const int64_t i = long_rows[ap.m - 1 - w];  // long rows fill the list from the back
     const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
     long long ub = 0;
     int lo = INT_MAX, hi = -1;
@@ -212,6 +225,32 @@ __global__ void __launch_bounds__(256) analyze_long_kernel(const RowPlan<T> p, c
       record_row(p, ap, i, e - s, ub, lo, hi, INT_MAX, s_seg, &s_prod, &s_slices, &s_empty);
     }
     __syncthreads();  // s_ub/s_lo/s_hi are reused by the next row
+  }
+  const int nmid = *reinterpret_cast<volatile int*>(&p.sum->n_mid);
+  const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t w = gw; w < nmid; w += nw) {
+    const int64_t i = long_rows[w];
+    const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
+    long long ub = 0;
+    int lo = INT_MAX, hi = -1;
+#pragma unroll 8
+    for (int64_t q = s + lane; q < e; q += 32) {
+      const int k = p.A.colidx[q];
+      const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];
+      if (be > bs) {
+        ub += be - bs;
+        lo = min(lo, p.B.colidx[bs]);
+        hi = max(hi, p.B.colidx[be - 1]);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      ub += __shfl_xor_sync(0xffffffffu, ub, o);
+      lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+      hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    }
+    if (lane == 0) record_row(p, ap, i, e - s, ub, lo, hi, INT_MAX, s_seg, &s_prod, &s_slices, &s_empty);
   }
   __syncthreads();
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
@@ -308,7 +347,7 @@ template <typename T>
 void launch_analyze(const RowPlan<T>& p, const AnalyzeParams& ap, int32_t* long_rows, const int32_t* rows,
                     int num_sms, cudaStream_t s, int* launches) {
   analyze_kernel<T><<<grid_for(ap.m, 256, num_sms, 8), 256, 0, s>>>(p, ap, long_rows, rows);
-  analyze_long_kernel<T><<<num_sms * 4, 256, 0, s>>>(p, ap, long_rows);
+  analyze_long_kernel<T><<<num_sms * 8, 256, 0, s>>>(p, ap, long_rows);
   *launches += 2;
 }
 

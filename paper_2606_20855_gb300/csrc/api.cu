@@ -36,7 +36,7 @@ int g_run_limit = 64;
 int g_dense_width = 0;  // 0 = default per value type
 int g_ewise_lanes = -1;  // elementwise: lanes per chunk (0 = lane groups from the mean row length, -1 = automatic)
 int64_t g_ewise_diag = 64;  // elementwise, one thread per chunk: merged positions per chunk
-constexpr int kLongRowThreshold = 128;
+constexpr int kLongRowThreshold = 16;  // rows with more stored entries are analysed by a warp or a CTA
 
 ws_status_t fail(ws_status_t st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
 ws_status_t fail(ws_status_t st, const char* fmt, ...) {

@@ -112,7 +112,8 @@ struct DevSummary {
   long long rcd_mega_entries;  // stored A entries of the dense heavy rows split into (row, slice) items
   int status;
   int n_sort;
-  int n_long;
+  int n_long;   // rows analysed by a CTA each (queued from the back of the long-row list)
+  int n_mid;    // rows analysed by a warp each (queued from the front)
   int n_empty;
   int bad_row;
   int n_pending;  // rows the planning pass left to the analysis kernel
