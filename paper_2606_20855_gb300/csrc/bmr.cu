@@ -361,7 +361,7 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
 
 // First pass over A when B has at most 65,536 columns: every row with
 // 2..bmr_max_a stored entries, a non-empty product, B rows that fit one group
-// and a bitmap of at most 8 words per product is ranked right here (class
+// and a bitmap of at most kPlanWordsPerProduct words per product is ranked right here (class
 // kClsBmrWide, lo = 0); every other row goes to `pending` for the analysis
 // kernel.  Counts per class are added to the summary.
 //
@@ -375,6 +375,11 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
 // the first column of each of its words.  A product's rank is then that word
 // rank plus the bits below it in its word.
 constexpr int kPlanThreads = 64;
+// Sparsest row the planning pass takes: its sweep and clear cost the same for
+// every row of a launch (the whole bitmap), so rows with fewer products go to
+// the hash bins, whose cost follows the product count.  At 16 words per
+// product a 65,536-column bitmap takes rows of 124 products and more.
+constexpr long long kPlanWordsPerProduct = 16;
 
 template <int LOGW>
 struct PlanShape {
@@ -470,7 +475,7 @@ __global__ void __launch_bounds__(kPlanThreads, kPlanMinBlocks) bmr_plan_kernel(
         ub += s_red[w2];
         mx = max(mx, s_red[kW + w2]);
       }
-      ok = ub > 0 && mx <= G && words <= 8ll * ub + 64;
+      ok = ub > 0 && mx <= G && words <= kPlanWordsPerProduct * static_cast<long long>(ub) + 64;
       if (ok) {
         // products of this thread: step s covers A entry j = s * kGroups + grp
         int col[kSteps];
