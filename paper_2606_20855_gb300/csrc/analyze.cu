@@ -75,19 +75,17 @@ __device__ __forceinline__ int segment_of(uint8_t cls) {
   return kSegHash0 + (cls - kClsHash0);                            // hash bins
 }
 
+// Stores the class and column range of row i (and its count if it is known
+// already) and returns the class.
 template <typename T>
-__device__ __forceinline__ void record_row(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t i, long long nnza,
-                                           long long ub, int lo, int hi, int maxlen, int* s_seg, long long* s_prod,
-                                           long long* s_slices, int* s_empty) {
+__device__ __forceinline__ uint8_t store_row(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t i, long long nnza,
+                                             long long ub, int lo, int hi, int maxlen, long long* s_slices) {
   const uint8_t c = classify(nnza, ub, lo, hi, maxlen, ap);
   p.cls[i] = c;
   // Direct rows know their count already; the others start at 0 and are
   // filled by the hash / dense-window symbolic kernels.
   p.c_rowptr[i + 1] = (c == kClsDirect) ? ub : 0;
-  if (c == kClsEmpty) {
-    atomicAdd(s_empty, 1);
-  } else {
-    atomicAdd(&s_seg[segment_of(c)], 1);
+  if (c != kClsEmpty) {
     p.lo[i] = lo;
     p.hi[i] = hi;
     if (c == kClsDense) {
@@ -95,6 +93,21 @@ __device__ __forceinline__ void record_row(const RowPlan<T>& p, const AnalyzePar
       atomicAdd(reinterpret_cast<unsigned long long*>(s_slices),
                 static_cast<unsigned long long>((span + ap.dense_width - 1) / ap.dense_width));
     }
+  }
+  return c;
+}
+
+// store_row for one row analysed by a single thread, with its counts added
+// to the CTA's counters.
+template <typename T>
+__device__ __forceinline__ void record_row(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t i, long long nnza,
+                                           long long ub, int lo, int hi, int maxlen, int* s_seg, long long* s_prod,
+                                           long long* s_slices, int* s_empty) {
+  const uint8_t c = store_row(p, ap, i, nnza, ub, lo, hi, maxlen, s_slices);
+  if (c == kClsEmpty) {
+    atomicAdd(s_empty, 1);
+  } else {
+    atomicAdd(&s_seg[segment_of(c)], 1);
   }
   atomicAdd(reinterpret_cast<unsigned long long*>(s_prod), static_cast<unsigned long long>(ub));
 }
@@ -133,33 +146,55 @@ __global__ void __launch_bounds__(256) analyze_kernel(const RowPlan<T> p, const 
   }
   __syncthreads();
   const int64_t nrows = rows ? static_cast<int64_t>(*reinterpret_cast<volatile int*>(&p.sum->n_pending)) : ap.m;
-  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < nrows;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t i = rows ? rows[t] : t;
-    const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
-    if (e - s > ap.long_threshold) {
-      if (e - s <= kMidRowMax) {
-        long_rows[atomicAdd(&p.sum->n_mid, 1)] = static_cast<int32_t>(i);
+  // Whole warps walk the rows (lane l takes row t0 + l), so that the counts
+  // per class can be added once per warp and class: every row adding to the
+  // same few CTA counters serialised on the shared-memory atomics.
+  const int lane = threadIdx.x & 31;
+  unsigned long long prod = 0;
+  for (int64_t t0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); t0 < nrows;
+       t0 += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t t = t0 + lane;
+    int seg = -2;  // no row, or a long row (queued)
+    if (t < nrows) {
+      const int64_t i = rows ? rows[t] : t;
+      const int64_t s = p.A.rowptr[i], e = p.A.rowptr[i + 1];
+      if (e - s > ap.long_threshold) {
+        if (e - s <= kMidRowMax) {
+          long_rows[atomicAdd(&p.sum->n_mid, 1)] = static_cast<int32_t>(i);
+        } else {
+          long_rows[ap.m - 1 - atomicAdd(&p.sum->n_long, 1)] = static_cast<int32_t>(i);
+        }
       } else {
-        long_rows[ap.m - 1 - atomicAdd(&p.sum->n_long, 1)] = static_cast<int32_t>(i);
-      }
-      continue;
-    }
-    long long ub = 0;
-    int lo = INT_MAX, hi = -1, maxlen = 0;
+        long long ub = 0;
+        int lo = INT_MAX, hi = -1, maxlen = 0;
 #pragma unroll 4
-    for (int64_t q = s; q < e; ++q) {
-      const int k = p.A.colidx[q];
-      const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];
-      if (be > bs) {
-        ub += be - bs;
-        maxlen = max(maxlen, static_cast<int>(min(be - bs, static_cast<int64_t>(INT_MAX))));
-        lo = min(lo, p.B.colidx[bs]);
-        hi = max(hi, p.B.colidx[be - 1]);
+        for (int64_t q = s; q < e; ++q) {
+          const int k = p.A.colidx[q];
+          const int64_t bs = p.B.rowptr[k], be = p.B.rowptr[k + 1];
+          if (be > bs) {
+            ub += be - bs;
+            maxlen = max(maxlen, static_cast<int>(min(be - bs, static_cast<int64_t>(INT_MAX))));
+            lo = min(lo, p.B.colidx[bs]);
+            hi = max(hi, p.B.colidx[be - 1]);
+          }
+        }
+        const uint8_t c = store_row(p, ap, i, e - s, ub, lo, hi, maxlen, &s_slices);
+        seg = c == kClsEmpty ? -1 : segment_of(c);
+        prod += static_cast<unsigned long long>(ub);
       }
     }
-    record_row(p, ap, i, e - s, ub, lo, hi, maxlen, s_seg, &s_prod, &s_slices, &s_empty);
+    const unsigned peers = __match_any_sync(0xffffffffu, seg);
+    if (seg >= -1 && lane == __ffs(peers) - 1) {
+      if (seg < 0) {
+        atomicAdd(&s_empty, __popc(peers));
+      } else {
+        atomicAdd(&s_seg[seg], __popc(peers));
+      }
+    }
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) prod += __shfl_xor_sync(0xffffffffu, prod, o);
+  if (lane == 0 && prod) atomicAdd(reinterpret_cast<unsigned long long*>(&s_prod), prod);
   __syncthreads();
   flush_counts(p, s_seg, &s_prod, &s_slices, &s_empty);
 }

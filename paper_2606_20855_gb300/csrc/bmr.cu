@@ -179,33 +179,92 @@ __device__ __forceinline__ int rank_products(uint32_t* bm, uint32_t* sm, uint16_
   return total;
 }
 
+// Symbolic pass of the binned register bitmap rows.  Like the numeric pass
+// below, a warp takes kHdrRows rows of its share at a time: the lanes first
+// fetch, for all of them together, the row bounds, the row's first column and
+// every stored A entry with its B row extent (the chain of dependent loads is
+// paid once per batch), then rank the rows one by one, each with one round of
+// independent loads of its products.
+constexpr int kHdrRows = 8;
+
+template <int LOGW>
+constexpr size_t symbolic_warp_bytes() {
+  return BmrShape<LOGW>::bytes() + static_cast<size_t>(kHdrRows) * kBmrMaxA * (sizeof(long long) + sizeof(int)) +
+         static_cast<size_t>(kHdrRows) * 2 * sizeof(int);
+}
+
 template <typename T, int LOGW, int G>
-__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const RowPlan<T> p) {
+__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const RowPlan<T> p, int hb) {
   using S = BmrShape<LOGW>;
-  constexpr int kSteps = kBmrMaxA / (32 / G);
+  constexpr int kGroups = 32 / G;
+  constexpr int kSteps = kBmrMaxA / kGroups;
+  constexpr int kEnt = kHdrRows * kBmrMaxA;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * S::bytes();
+  const int grp = lane / G, gl = lane % G;
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * symbolic_warp_bytes<LOGW>();
   uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
   uint16_t* pre = reinterpret_cast<uint16_t*>(ws + static_cast<size_t>(S::kPhysWords) * 4);
   int* base = reinterpret_cast<int*>(ws + static_cast<size_t>(S::kPhysWords) * 6);
   uint32_t* sm = reinterpret_cast<uint32_t*>(base + 32);
+  long long* h_b0 = reinterpret_cast<long long*>(ws + S::bytes());
+  int* h_len = reinterpret_cast<int*>(h_b0 + kEnt);
+  int* h_row = h_len + kEnt;
+  int* h_lo = h_row + kHdrRows;
   for (int s2 = lane; s2 < S::kPhysWords; s2 += 32) bm[s2] = 0u;
   for (int s2 = lane; s2 < S::kSPL * 32; s2 += 32) sm[s2] = 0u;
   __syncwarp();
 
-  for (int64_t r = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub; r < p.seg_len;
-       r += static_cast<int64_t>(gridDim.x) * kRowsPerCta) {
-    const int32_t row = p.perm[p.seg_begin + r];
-    const int64_t ra = p.A.rowptr[row];
-    const int na = static_cast<int>(p.A.rowptr[row + 1] - ra);
-    int col[kSteps];
-    T val[kSteps];
-    load_products<T, G, false, kSteps>(p, ra, na, lane, col, val);
-    const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, p.lo[row], lane,
-                                               p.ranks + static_cast<int64_t>(row) * kBmrSlots);
-    if (lane == 0) p.c_rowptr[row + 1] = total;
+  // hb (1..kHdrRows) rows per batch: fewer when the segment is too short to
+  // give every warp of the grid a full batch.
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
+  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * hb; r0 < p.seg_len; r0 += warps * hb) {
+    // Batch header: lane i < hb fetches row r0 + i.
+    int na_l = 0;
+    long long ra_l = 0;
+    if (lane < kHdrRows) {
+      int row_l = -1;
+      if (lane < hb && r0 + lane < p.seg_len) {
+        row_l = p.perm[p.seg_begin + r0 + lane];
+        ra_l = p.A.rowptr[row_l];
+        const long long na = p.A.rowptr[row_l + 1] - ra_l;
+        na_l = static_cast<int>(na < kBmrMaxA ? (na > 0 ? na : 0) : kBmrMaxA);
+        h_lo[lane] = p.lo[row_l];
+      }
+      h_row[lane] = row_l;
+    }
+#pragma unroll
+    for (int q = 0; q < kEnt / 32; ++q) {
+      const int e = q * 32 + lane;
+      const int i = e / kBmrMaxA, j = e % kBmrMaxA;
+      const long long ra = __shfl_sync(kFull, ra_l, i);
+      const int na = __shfl_sync(kFull, na_l, i);
+      int len = 0;
+      if (j < na) {
+        const int k = p.A.colidx[ra + j];
+        const long long b0 = p.B.rowptr[k];
+        len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        h_b0[e] = b0;
+      }
+      h_len[e] = len;
+    }
+    __syncwarp();
+    for (int i = 0; i < kHdrRows; ++i) {
+      const int row = h_row[i];
+      if (row < 0) break;
+      int col[kSteps];
+#pragma unroll
+      for (int st = 0; st < kSteps; ++st) {
+        const int e = i * kBmrMaxA + st * kGroups + grp;
+        col[st] = -1;
+        if (gl < h_len[e]) col[st] = p.B.colidx[h_b0[e] + gl];
+      }
+      const int total = rank_products<S, kSteps>(bm, sm, pre, base, col, h_lo[i], lane,
+                                                 p.ranks + static_cast<int64_t>(row) * kBmrSlots);
+      if (lane == 0) p.c_rowptr[row + 1] = total;
+    }
+    __syncwarp();  // the next batch rewrites the headers
   }
 }
 
@@ -218,7 +277,6 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const
 // its column and value at its rank in a compact staging array, the products
 // that repeat a column add theirs (a shared-memory atomic, the atomic level
 // of Sec. 4), and the warp copies the sorted row to C with coalesced stores.
-constexpr int kHdrRows = 8;
 
 // Staging slots of one warp: a row has at most kBmrMaxA * G products (the
 // lane groups of G lanes take kBmrMaxA stored A entries), so at most that
@@ -651,11 +709,15 @@ void launch_bmr_g(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s
     bmr_numeric_kernel<T, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p, static_cast<int>(hb));
     return;
   }
-  const size_t smem = static_cast<size_t>(kRowsPerCta) * BmrShape<LOGW>::bytes();
+  const size_t smem = static_cast<size_t>(kRowsPerCta) * symbolic_warp_bytes<LOGW>();
   static int per_sm = 0;
   if (per_sm == 0) per_sm = occupancy(bmr_symbolic_kernel<T, LOGW, G>, 32 * kRowsPerCta, smem);
-  const int64_t grid = clamp_grid((p.seg_len + kRowsPerCta - 1) / kRowsPerCta, num_sms, per_sm);
-  bmr_symbolic_kernel<T, LOGW, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p);
+  const int64_t wave_warps = static_cast<int64_t>(num_sms) * per_sm * kRowsPerCta;
+  int64_t hb = (p.seg_len + wave_warps - 1) / wave_warps;
+  hb = hb < 1 ? 1 : (hb > kHdrRows ? kHdrRows : hb);
+  const int64_t per_cta = static_cast<int64_t>(kRowsPerCta) * hb;
+  const int64_t grid = clamp_grid((p.seg_len + per_cta - 1) / per_cta, num_sms, per_sm);
+  bmr_symbolic_kernel<T, LOGW, G><<<static_cast<int>(grid), 32 * kRowsPerCta, smem, s>>>(p, static_cast<int>(hb));
 }
 
 template <typename T, int LOGW>
