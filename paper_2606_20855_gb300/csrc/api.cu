@@ -187,7 +187,6 @@ struct Plan {
   int64_t seg_offset[kNumSegs + 1] = {};
   int64_t n_sort = 0, n_empty = 0, dense_slices = 0, products = 0;
   int log2_group = 5;
-  int wide_bin = 2;  // register bitmap bin of the rows counted by the planning pass
   bool all_planned = false;  // the planning pass took every row: its segment is rows 0..m-1 in order
   int dense_width = 0;
   int run_limit = 64;
@@ -421,7 +420,6 @@ ws_status_t symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Pla
     // 65,536 columns), the planning pass counts the eligible rows in its first
     // read of A and only the remaining rows go through the analysis kernel.
     const bool plan_pass = g_bmr_max_a > 0 && B->ncols > 0 && B->ncols <= kMaxBitmapSpan && g_bitmap_span >= B->ncols;
-    pl->wide_bin = bmr_bin_for_span(B->ncols);
     if (plan_pass) {
       st = pl->ranks.reserve(static_cast<size_t>(m) * kBmrSlots * sizeof(uint16_t), s);
       if (st != WS_OK) return st;
@@ -483,7 +481,7 @@ ws_status_t numeric_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, Plan
     p.seg_begin = pl->seg_offset[kSegBmrWide];
     p.seg_len = pl->seg_count[kSegBmrWide];
     if (pl->all_planned) p.perm = nullptr;  // rows in order, no permutation was built
-    launch_bmr<T>(p, pl->wide_bin, true, sms, s, &pl->num_launches);
+    launch_bmr<T>(p, kBmrPlannedBin, true, sms, s, &pl->num_launches);
     p.perm = pl->perm;
   }
   if (pl->seg_count[kSegRcd] > 0) {

@@ -417,6 +417,275 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
   }
 }
 
+// Grouped register bitmap rows: bin 0 (column range of at most kGrpWords * 32
+// columns) when B's rows fit groups of G <= 8 lanes.  A row of a few short B
+// rows (a stencil row: 5 stored entries of 5 products each) leaves most of a
+// warp idle and pays the warp's fixed per-row work (headers, scan, sweep,
+// copy-out) for a handful of products, so here each group of G lanes owns a
+// row and a warp ranks 32 / G rows at once.  Lane gl of group g takes element
+// gl of every B row of the group's row (step st = stored A entry st).
+//
+// Bitmap: the row of group g has kGrpWords words; lane g*G + i owns words
+// [i * WPL, (i + 1) * WPL) (WPL = kGrpWords / G <= 32), and word w sits at
+// (w % WPL) * 32 + owner lane, so each lane's words are in its own bank and
+// one summary word per lane marks which of them are non-zero.  The ranks of
+// a row are stored as uint16 at slot st * G + gl.
+constexpr int kGrpLogW = 7;
+constexpr int kGrpWords = 1 << kGrpLogW;
+static_assert(32 << kGrpLogW == 32 << bmr_log_words(0), "grouped rows are the rows of bin 0");
+
+template <int G>
+struct GrpShape {
+  static constexpr int kRows = 32 / G;          // rows per warp
+  static constexpr int kWPL = kGrpWords / G;    // bitmap words per lane
+  static constexpr int kPhys = kWPL * 32;       // bitmap words per warp
+  static_assert(kWPL <= 32, "one summary word per lane");
+  static constexpr int kEnt = kRows * kBmrMaxA;  // stored A entries per warp
+};
+
+template <int G>
+constexpr size_t grp_symbolic_warp_bytes() {
+  using S = GrpShape<G>;
+  return static_cast<size_t>(S::kPhys) * 6 + 32 * 4 * 2 + static_cast<size_t>(S::kEnt) * (sizeof(long long) + sizeof(int));
+}
+
+template <typename T, int G>
+__global__ void __launch_bounds__(32 * kRowsPerCta, 8) bmr_group_symbolic_kernel(const RowPlan<T> p) {
+  using S = GrpShape<G>;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int sub = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int g = lane / G, gl = lane % G;
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * grp_symbolic_warp_bytes<G>();
+  uint32_t* bm = reinterpret_cast<uint32_t*>(ws);
+  uint16_t* pre = reinterpret_cast<uint16_t*>(bm + S::kPhys);
+  uint32_t* sm = reinterpret_cast<uint32_t*>(pre + S::kPhys);
+  int* base = reinterpret_cast<int*>(sm + 32);
+  long long* h_b0 = reinterpret_cast<long long*>(base + 32) + g * kBmrMaxA;
+  int* h_len = reinterpret_cast<int*>(reinterpret_cast<long long*>(base + 32) + S::kEnt) + g * kBmrMaxA;
+  for (int i = lane; i < S::kPhys; i += 32) bm[i] = 0u;
+  sm[lane] = 0u;
+  __syncwarp();
+
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
+  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * S::kRows; r0 < p.seg_len;
+       r0 += warps * S::kRows) {
+    const int64_t r = r0 + g;
+    int row = -1, na = 0, lo = 0;
+    long long ra = 0;
+    if (r < p.seg_len) {
+      row = p.perm[p.seg_begin + r];
+      ra = p.A.rowptr[row];
+      const long long n = p.A.rowptr[row + 1] - ra;
+      na = static_cast<int>(n < kBmrMaxA ? n : kBmrMaxA);
+      lo = p.lo[row];
+    }
+#pragma unroll
+    for (int jj = 0; jj < kBmrMaxA / G; ++jj) {
+      const int j = jj * G + gl;
+      int len = 0;
+      if (j < na) {
+        const int k = p.A.colidx[ra + j];
+        const long long b0 = p.B.rowptr[k];
+        len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        h_b0[j] = b0;
+      }
+      h_len[j] = len;
+    }
+    int nmax = na;
+#pragma unroll
+    for (int o = 16; o >= G; o >>= 1) nmax = max(nmax, __shfl_xor_sync(kFull, nmax, o));
+    __syncwarp();
+    int col[kBmrMaxA];
+#pragma unroll
+    for (int st = 0; st < kBmrMaxA; ++st) {
+      col[st] = -1;
+      if (st < nmax && st < na && gl < h_len[st]) col[st] = p.B.colidx[h_b0[st] + gl];
+    }
+    uint32_t dup = 0;
+#pragma unroll
+    for (int st = 0; st < kBmrMaxA; ++st) {
+      if (st < nmax && col[st] >= 0) {
+        const uint32_t w = static_cast<uint32_t>(col[st] - lo) >> 5;
+        const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
+        const uint32_t j = w % S::kWPL;
+        const uint32_t bit = 1u << ((col[st] - lo) & 31);
+        if (atomicOr(bm + ((j << 5) | owner), bit) & bit) dup |= 1u << st;
+        atomicOr(sm + owner, 1u << j);
+      }
+    }
+    __syncwarp();
+    // Rank of the first column of each non-zero word this lane owns.
+    uint32_t m = sm[lane];
+    sm[lane] = 0u;
+    int run = 0;
+    while (m) {
+      const int b = __ffs(m) - 1;
+      m &= m - 1u;
+      const int ph = (b << 5) | lane;
+      pre[ph] = static_cast<uint16_t>(run);
+      run += __popc(bm[ph]);
+    }
+    // Exclusive scan over the G lanes of the group (word order = lane order).
+    int incl = run;
+#pragma unroll
+    for (int o = 1; o < G; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, incl, o, G);
+      if (gl >= o) incl += y;
+    }
+    base[lane] = incl - run;
+    const int total = __shfl_sync(kFull, incl, G - 1, G);
+    __syncwarp();
+    uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
+#pragma unroll
+    for (int st = 0; st < kBmrMaxA; ++st) {
+      if (st < nmax && col[st] >= 0) {
+        const uint32_t off = static_cast<uint32_t>(col[st] - lo);
+        const uint32_t w = off >> 5;
+        const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
+        const uint32_t ph = ((w % S::kWPL) << 5) | owner;
+        const int pos = base[owner] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
+        ranks[st * G + gl] = static_cast<uint16_t>(pos | static_cast<int>(((dup >> st) & 1u) << 15));
+      }
+    }
+    __syncwarp();
+#pragma unroll
+    for (int st = 0; st < kBmrMaxA; ++st) {
+      if (st < nmax && col[st] >= 0) {
+        const uint32_t w = static_cast<uint32_t>(col[st] - lo) >> 5;
+        bm[((w % S::kWPL) << 5) | (static_cast<uint32_t>(g * G) + w / S::kWPL)] = 0u;
+      }
+    }
+    if (gl == 0 && row >= 0) p.c_rowptr[row + 1] = total;
+    __syncwarp();
+  }
+}
+
+// Numeric pass of the grouped rows: group g places its row's products at
+// their stored ranks in its own staging array (first product of a column
+// stores, repeats add afterwards) and copies the sorted row to C.
+template <typename T, int G>
+constexpr size_t grp_numeric_warp_bytes() {
+  using S = GrpShape<G>;
+  return static_cast<size_t>(S::kRows) * kBmrMaxA * G * (4 + sizeof(T)) +
+         static_cast<size_t>(S::kEnt) * (sizeof(long long) + sizeof(T) + sizeof(int));
+}
+
+template <typename T, int G>
+__global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(const RowPlan<T> p) {
+  using S = GrpShape<G>;
+  constexpr int kCap = kBmrMaxA * G;  // products (so entries) of a row at most
+  constexpr int kHalf = kBmrMaxA / 2;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int sub = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int g = lane / G, gl = lane % G;
+  // Per warp: staging values and columns of every group, then the stored A
+  // entries of every group (B row start, A value, B row length).
+  unsigned char* ws = smem_raw + static_cast<size_t>(sub) * grp_numeric_warp_bytes<T, G>();
+  constexpr size_t kKeyOff = static_cast<size_t>(S::kRows) * kCap * sizeof(T);
+  constexpr size_t kB0Off = kKeyOff + static_cast<size_t>(S::kRows) * kCap * 4;
+  constexpr size_t kAOff = kB0Off + static_cast<size_t>(S::kEnt) * sizeof(long long);
+  constexpr size_t kLenOff = kAOff + static_cast<size_t>(S::kEnt) * sizeof(T);
+  T* st_val = reinterpret_cast<T*>(ws) + g * kCap;
+  int* st_key = reinterpret_cast<int*>(ws + kKeyOff) + g * kCap;
+  long long* h_b0 = reinterpret_cast<long long*>(ws + kB0Off) + g * kBmrMaxA;
+  T* h_a = reinterpret_cast<T*>(ws + kAOff) + g * kBmrMaxA;
+  int* h_len = reinterpret_cast<int*>(ws + kLenOff) + g * kBmrMaxA;
+
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
+  for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * S::kRows; r0 < p.seg_len;
+       r0 += warps * S::kRows) {
+    const int64_t r = r0 + g;
+    int row = -1, na = 0;
+    long long ra = 0, cbase = 0, want = 0;
+    if (r < p.seg_len) {
+      row = p.perm[p.seg_begin + r];
+      ra = p.A.rowptr[row];
+      const long long n = p.A.rowptr[row + 1] - ra;
+      na = static_cast<int>(n < kBmrMaxA ? n : kBmrMaxA);
+      cbase = p.c_rowptr[row];
+      want = p.c_rowptr[row + 1] - cbase;
+    }
+    const int cnt = static_cast<int>(want < kCap ? want : kCap);  // staging bounds every access
+    bool bad = want > kCap;
+#pragma unroll
+    for (int jj = 0; jj < kBmrMaxA / G; ++jj) {
+      const int j = jj * G + gl;
+      int len = 0;
+      if (j < na) {
+        const int k = p.A.colidx[ra + j];
+        const long long b0 = p.B.rowptr[k];
+        len = static_cast<int>(p.B.rowptr[k + 1] - b0);
+        h_b0[j] = b0;
+        h_a[j] = p.A.vals[ra + j];
+      }
+      h_len[j] = len;
+    }
+    int nmax = na;
+#pragma unroll
+    for (int o = 16; o >= G; o >>= 1) nmax = max(nmax, __shfl_xor_sync(kFull, nmax, o));
+    __syncwarp();
+    const uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
+    uint32_t repeats = 0;
+    // Two halves of eight steps: all loads of a half are in flight before
+    // its products are placed.
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (h * kHalf < nmax) {
+        int col[kHalf], rk[kHalf];
+        T val[kHalf];
+#pragma unroll
+        for (int u = 0; u < kHalf; ++u) {
+          const int st = h * kHalf + u;
+          col[u] = -1;
+          rk[u] = 0;
+          val[u] = T(0);
+          if (st < na && gl < h_len[st]) {
+            const long long q = h_b0[st] + gl;
+            col[u] = p.B.colidx[q];
+            val[u] = p.B.vals[q];
+            rk[u] = ranks[st * G + gl];
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kHalf; ++u) {
+          if (col[u] >= 0) {
+            const int st = h * kHalf + u;
+            const int rr = rk[u] & 0x7fff;
+            if (rr >= cnt) {
+              bad = true;
+            } else if (rk[u] & 0x8000) {
+              repeats |= 1u << st;
+            } else {
+              st_key[rr] = col[u];
+              st_val[rr] = h_a[st] * val[u];
+            }
+          }
+        }
+      }
+    }
+    if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
+    __syncwarp();
+    if (__any_sync(kFull, repeats != 0)) {
+      // products whose column another product of the row placed: add theirs
+      while (repeats) {
+        const int st = __ffs(repeats) - 1;
+        repeats &= repeats - 1u;
+        const long long q = h_b0[st] + gl;
+        const int rr = ranks[st * G + gl] & 0x7fff;
+        atomicAdd(&st_val[rr], h_a[st] * p.B.vals[q]);
+      }
+      __syncwarp();
+    }
+    for (int s2 = gl; s2 < cnt; s2 += G) {
+      p.c_colidx[cbase + s2] = st_key[s2];
+      p.c_vals[cbase + s2] = st_val[s2];
+    }
+    __syncwarp();
+  }
+}
+
 // First pass over A when B has at most 65,536 columns: every row with
 // 2..bmr_max_a stored entries, a non-empty product, B rows that fit one group
 // and a bitmap of at most kPlanWordsPerProduct words per product is ranked right here (class
@@ -740,14 +1009,45 @@ void launch_plan_g(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, 
   bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), kPlanThreads, smem, s>>>(p, ap, ncols, pending);
 }
 
+template <typename T, int G>
+void launch_grp(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s) {
+  constexpr int64_t kPerCta = static_cast<int64_t>(kRowsPerCta) * GrpShape<G>::kRows;
+  const int64_t want = (p.seg_len + kPerCta - 1) / kPerCta;
+  if (numeric) {
+    const size_t smem = static_cast<size_t>(kRowsPerCta) * grp_numeric_warp_bytes<T, G>();
+    static int per_sm = 0;
+    if (per_sm == 0) per_sm = occupancy(bmr_group_numeric_kernel<T, G>, 32 * kRowsPerCta, smem);
+    bmr_group_numeric_kernel<T, G>
+        <<<static_cast<int>(clamp_grid(want, num_sms, per_sm)), 32 * kRowsPerCta, smem, s>>>(p);
+  } else {
+    const size_t smem = static_cast<size_t>(kRowsPerCta) * grp_symbolic_warp_bytes<G>();
+    static int per_sm = 0;
+    if (per_sm == 0) per_sm = occupancy(bmr_group_symbolic_kernel<T, G>, 32 * kRowsPerCta, smem);
+    bmr_group_symbolic_kernel<T, G>
+        <<<static_cast<int>(clamp_grid(want, num_sms, per_sm)), 32 * kRowsPerCta, smem, s>>>(p);
+  }
+}
+
 }  // namespace
 
 template <typename T>
 void launch_bmr(const RowPlan<T>& p, int bin, bool numeric, int num_sms, cudaStream_t s, int* launches) {
+  if (bin == 0 && p.log2_group <= 3) {  // B rows of at most 8 entries: a group of lanes per row
+    if (p.log2_group == 2) {
+      launch_grp<T, 4>(p, numeric, num_sms, s);
+    } else {
+      launch_grp<T, 8>(p, numeric, num_sms, s);
+    }
+    *launches += 1;
+    return;
+  }
   switch (bin) {
     case 0: launch_bmr_w<T, bmr_log_words(0)>(p, numeric, num_sms, s); break;
     case 1: launch_bmr_w<T, bmr_log_words(1)>(p, numeric, num_sms, s); break;
     case 2: launch_bmr_w<T, bmr_log_words(2)>(p, numeric, num_sms, s); break;
+    case kBmrPlannedBin:  // ranked by the planning pass in the one-warp layout
+      if (numeric) launch_bmr_w<T, bmr_log_words(0)>(p, true, num_sms, s);
+      break;
     default: return;
   }
   *launches += 1;

@@ -48,12 +48,14 @@ __host__ __device__ constexpr int bitmap_cap(int b) {
 }
 
 // Register bitmap bins: rows with at most kBmrMaxA stored A entries whose B
-// rows fit one lane group; bitmap of 1 << kBmrLogWords[b] words.
+// rows fit one lane group; bitmap of 1 << bmr_log_words(b) words (column
+// ranges of at most 4096, 16,384 and 65,536 columns).
 constexpr int kNumBmrBins = 3;
+constexpr int kBmrPlannedBin = kNumBmrBins;  // launch_bmr: numeric pass of the rows ranked by the planning pass
 constexpr int kBmrMaxA = 16;
 constexpr int kBmrCap = 512;  // >= kBmrMaxA * 32 products
 constexpr int kBmrSlots = 512;  // rank slots per register bitmap row (one per possible product)
-__host__ __device__ constexpr int bmr_log_words(int b) { return b == 0 ? 6 : b == 1 ? 9 : 11; }
+__host__ __device__ constexpr int bmr_log_words(int b) { return b == 0 ? 7 : b == 1 ? 9 : 11; }
 // Smallest register bitmap bin whose bitmap covers `span` columns (span <= kMaxBitmapSpan).
 __host__ __device__ constexpr int bmr_bin_for_span(long long span) {
   return span <= (32ll << bmr_log_words(0)) ? 0 : span <= (32ll << bmr_log_words(1)) ? 1 : 2;

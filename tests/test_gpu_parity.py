@@ -59,6 +59,44 @@ def test_uniform_several_tiles(dtype, path):
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
+def _banded(m, n, lens, halfwidth, rng, dtype, centre):
+    """Rows of the given lengths with distinct columns within halfwidth of centre(i)."""
+    rows = {}
+    for i, L in enumerate(lens):
+        c = int(centre(i))
+        lo, hi = max(0, c - halfwidth), min(n, c + halfwidth + 1)
+        L = min(L, hi - lo)
+        rows[i] = (lo + rng.choice(hi - lo, size=L, replace=False)).tolist()
+    M = _csr(m, n, rows, dtype=dtype)
+    M.vals = (2 * rng.random(M.nnz) - 1).astype(dtype)
+    return M
+
+
+@pytest.mark.parametrize("b_len", [4, 8])
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_grouped_register_rows(dtype, b_len):
+    """Banded products over more than 65,536 columns whose B rows fit 4 or 8
+    lanes: rows of at most 4096 columns are ranked by groups of lanes, several
+    rows per warp, with stored-entry counts 0..16 mixed inside every warp,
+    repeated columns, a ragged last warp, and wider rows (other bins) between
+    them."""
+    rng = np.random.default_rng(40 + b_len)
+    k = n = 100_000
+    B = _banded(k, n, [b_len] * k, 600, rng, dtype, lambda j: j)
+    m = 20_011
+    lens = rng.integers(0, 17, size=m)
+    A = _banded(m, k, lens, 700, rng, dtype, lambda i: i * (k // m))
+    wide = rng.choice(m, size=200, replace=False)  # rows spread over a wider range
+    rows = {i: A.colidx[A.rowptr[i]:A.rowptr[i + 1]].tolist() for i in range(m)}
+    for i in wide:
+        L = int(rng.integers(2, 17))
+        rows[int(i)] = rng.choice(k, size=L, replace=False).tolist()
+    A = _csr(m, k, rows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    rowptr, colidx, vals, info = run_gpu(A, B, validate=True)
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+
+
 @pytest.mark.parametrize("dtype", DTYPES)
 @pytest.mark.parametrize("n", [2_000, 16_000, 60_000])
 def test_bitmap_bins(dtype, n):
