@@ -432,6 +432,7 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
 // a row are stored as uint16 at slot st * G + gl.
 constexpr int kGrpLogW = 7;
 constexpr int kGrpWords = 1 << kGrpLogW;
+constexpr int kGrpChunk = 4;  // steps per warp-uniform branch
 static_assert(32 << kGrpLogW == 32 << bmr_log_words(0), "grouped rows are the rows of bin 0");
 
 template <int G>
@@ -496,27 +497,41 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 8) bmr_group_symbolic_kernel
 #pragma unroll
     for (int o = 16; o >= G; o >>= 1) nmax = max(nmax, __shfl_xor_sync(kFull, nmax, o));
     __syncwarp();
+    // Steps in chunks of kGrpChunk behind warp-uniform branches: a stencil
+    // row has 5 stored entries, so most of the 16 steps are skipped.
     int col[kBmrMaxA];
 #pragma unroll
-    for (int st = 0; st < kBmrMaxA; ++st) {
-      col[st] = -1;
-      if (st < nmax && st < na && gl < h_len[st]) col[st] = p.B.colidx[h_b0[st] + gl];
-    }
+    for (int st = 0; st < kBmrMaxA; ++st) col[st] = -1;
     uint32_t dup = 0;
 #pragma unroll
-    for (int st = 0; st < kBmrMaxA; ++st) {
-      if (st < nmax && col[st] >= 0) {
-        const uint32_t w = static_cast<uint32_t>(col[st] - lo) >> 5;
-        const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
-        const uint32_t j = w % S::kWPL;
-        const uint32_t bit = 1u << ((col[st] - lo) & 31);
-        if (atomicOr(bm + ((j << 5) | owner), bit) & bit) dup |= 1u << st;
-        atomicOr(sm + owner, 1u << j);
+    for (int c = 0; c < kBmrMaxA / kGrpChunk; ++c) {
+      if (c * kGrpChunk < nmax) {
+#pragma unroll
+        for (int u = 0; u < kGrpChunk; ++u) {
+          const int st = c * kGrpChunk + u;
+          if (st < na && gl < h_len[st]) col[st] = p.B.colidx[h_b0[st] + gl];
+        }
+#pragma unroll
+        for (int u = 0; u < kGrpChunk; ++u) {
+          const int st = c * kGrpChunk + u;
+          if (col[st] >= 0) {
+            const uint32_t w = static_cast<uint32_t>(col[st] - lo) >> 5;
+            const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
+            const uint32_t j = w % S::kWPL;
+            const uint32_t bit = 1u << ((col[st] - lo) & 31);
+            if (atomicOr(bm + ((j << 5) | owner), bit) & bit) dup |= 1u << st;
+            atomicOr(sm + owner, 1u << j);
+          }
+          // Steps in order: the product that keeps its column is the one of
+          // the lowest step (a group's lanes hold distinct columns within a step).
+          __syncwarp();
+        }
       }
     }
     __syncwarp();
     // Rank of the first column of each non-zero word this lane owns.
-    uint32_t m = sm[lane];
+    const uint32_t touched = sm[lane];
+    uint32_t m = touched;
     sm[lane] = 0u;
     int run = 0;
     while (m) {
@@ -538,32 +553,36 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 8) bmr_group_symbolic_kernel
     __syncwarp();
     uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
 #pragma unroll
-    for (int st = 0; st < kBmrMaxA; ++st) {
-      if (st < nmax && col[st] >= 0) {
-        const uint32_t off = static_cast<uint32_t>(col[st] - lo);
-        const uint32_t w = off >> 5;
-        const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
-        const uint32_t ph = ((w % S::kWPL) << 5) | owner;
-        const int pos = base[owner] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
-        ranks[st * G + gl] = static_cast<uint16_t>(pos | static_cast<int>(((dup >> st) & 1u) << 15));
+    for (int c = 0; c < kBmrMaxA / kGrpChunk; ++c) {
+      if (c * kGrpChunk < nmax) {
+#pragma unroll
+        for (int u = 0; u < kGrpChunk; ++u) {
+          const int st = c * kGrpChunk + u;
+          if (col[st] >= 0) {
+            const uint32_t off = static_cast<uint32_t>(col[st] - lo);
+            const uint32_t w = off >> 5;
+            const uint32_t owner = static_cast<uint32_t>(g * G) + w / S::kWPL;
+            const uint32_t ph = ((w % S::kWPL) << 5) | owner;
+            const int pos = base[owner] + pre[ph] + __popc(bm[ph] & ((1u << (off & 31u)) - 1u));
+            ranks[st * G + gl] = static_cast<uint16_t>(pos | static_cast<int>(((dup >> st) & 1u) << 15));
+          }
+        }
       }
     }
     __syncwarp();
-#pragma unroll
-    for (int st = 0; st < kBmrMaxA; ++st) {
-      if (st < nmax && col[st] >= 0) {
-        const uint32_t w = static_cast<uint32_t>(col[st] - lo) >> 5;
-        bm[((w % S::kWPL) << 5) | (static_cast<uint32_t>(g * G) + w / S::kWPL)] = 0u;
-      }
-    }
+    // Clear the non-zero words this lane owns.
+    for (uint32_t t2 = touched; t2; t2 &= t2 - 1u) bm[((__ffs(t2) - 1) << 5) | lane] = 0u;
     if (gl == 0 && row >= 0) p.c_rowptr[row + 1] = total;
     __syncwarp();
   }
 }
 
 // Numeric pass of the grouped rows: group g places its row's products at
-// their stored ranks in its own staging array (first product of a column
-// stores, repeats add afterwards) and copies the sorted row to C.
+// their stored ranks in its own staging array and copies the sorted row to C.
+// Steps are placed in order, so the product that stores a column (the one of
+// the lowest step) comes before every product that adds to it, and within a
+// step the lanes of a group write distinct slots: plain shared-memory adds, no
+// atomics (a Laplacian row repeats 12 of its 25 product columns).
 template <typename T, int G>
 constexpr size_t grp_numeric_warp_bytes() {
   using S = GrpShape<G>;
@@ -575,7 +594,6 @@ template <typename T, int G>
 __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(const RowPlan<T> p) {
   using S = GrpShape<G>;
   constexpr int kCap = kBmrMaxA * G;  // products (so entries) of a row at most
-  constexpr int kHalf = kBmrMaxA / 2;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -627,17 +645,16 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(
     for (int o = 16; o >= G; o >>= 1) nmax = max(nmax, __shfl_xor_sync(kFull, nmax, o));
     __syncwarp();
     const uint16_t* ranks = p.ranks + static_cast<int64_t>(row) * kBmrSlots;
-    uint32_t repeats = 0;
-    // Two halves of eight steps: all loads of a half are in flight before
-    // its products are placed.
+    // Chunks of kGrpChunk steps behind warp-uniform branches: all loads of a
+    // chunk are in flight before its products are placed.
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      if (h * kHalf < nmax) {
-        int col[kHalf], rk[kHalf];
-        T val[kHalf];
+    for (int c = 0; c < kBmrMaxA / kGrpChunk; ++c) {
+      if (c * kGrpChunk < nmax) {
+        int col[kGrpChunk], rk[kGrpChunk];
+        T val[kGrpChunk];
 #pragma unroll
-        for (int u = 0; u < kHalf; ++u) {
-          const int st = h * kHalf + u;
+        for (int u = 0; u < kGrpChunk; ++u) {
+          const int st = c * kGrpChunk + u;
           col[u] = -1;
           rk[u] = 0;
           val[u] = T(0);
@@ -649,35 +666,25 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(
           }
         }
 #pragma unroll
-        for (int u = 0; u < kHalf; ++u) {
+        for (int u = 0; u < kGrpChunk; ++u) {
           if (col[u] >= 0) {
-            const int st = h * kHalf + u;
+            const int st = c * kGrpChunk + u;
             const int rr = rk[u] & 0x7fff;
             if (rr >= cnt) {
               bad = true;
             } else if (rk[u] & 0x8000) {
-              repeats |= 1u << st;
+              st_val[rr] += h_a[st] * val[u];
             } else {
               st_key[rr] = col[u];
               st_val[rr] = h_a[st] * val[u];
             }
           }
+          __syncwarp();
         }
       }
     }
     if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
     __syncwarp();
-    if (__any_sync(kFull, repeats != 0)) {
-      // products whose column another product of the row placed: add theirs
-      while (repeats) {
-        const int st = __ffs(repeats) - 1;
-        repeats &= repeats - 1u;
-        const long long q = h_b0[st] + gl;
-        const int rr = ranks[st * G + gl] & 0x7fff;
-        atomicAdd(&st_val[rr], h_a[st] * p.B.vals[q]);
-      }
-      __syncwarp();
-    }
     for (int s2 = gl; s2 < cnt; s2 += G) {
       p.c_colidx[cbase + s2] = st_key[s2];
       p.c_vals[cbase + s2] = st_val[s2];
