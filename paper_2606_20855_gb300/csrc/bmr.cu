@@ -435,13 +435,19 @@ constexpr int kGrpWords = 1 << kGrpLogW;
 constexpr int kGrpChunk = 4;  // steps per warp-uniform branch
 static_assert(32 << kGrpLogW == 32 << bmr_log_words(0), "grouped rows are the rows of bin 0");
 
+// The per-group arrays (entry headers, staging) are padded so that the same
+// index of different groups falls in different banks: neighbouring rows of a
+// stencil hit the same ranks and steps at the same time.
 template <int G>
 struct GrpShape {
   static constexpr int kRows = 32 / G;          // rows per warp
   static constexpr int kWPL = kGrpWords / G;    // bitmap words per lane
   static constexpr int kPhys = kWPL * 32;       // bitmap words per warp
   static_assert(kWPL <= 32, "one summary word per lane");
-  static constexpr int kEnt = kRows * kBmrMaxA;  // stored A entries per warp
+  static constexpr int kHdr = kBmrMaxA + 1;     // entry-header stride of a group
+  static constexpr int kEnt = kRows * kHdr;     // entry-header slots per warp
+  static constexpr int kCap = kBmrMaxA * G;     // products (so entries) of a row at most
+  static constexpr int kPadBytes = 128 / kRows;  // staging stride beyond kCap entries, in bytes
 };
 
 template <int G>
@@ -462,8 +468,8 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 8) bmr_group_symbolic_kernel
   uint16_t* pre = reinterpret_cast<uint16_t*>(bm + S::kPhys);
   uint32_t* sm = reinterpret_cast<uint32_t*>(pre + S::kPhys);
   int* base = reinterpret_cast<int*>(sm + 32);
-  long long* h_b0 = reinterpret_cast<long long*>(base + 32) + g * kBmrMaxA;
-  int* h_len = reinterpret_cast<int*>(reinterpret_cast<long long*>(base + 32) + S::kEnt) + g * kBmrMaxA;
+  long long* h_b0 = reinterpret_cast<long long*>(base + 32) + g * S::kHdr;
+  int* h_len = reinterpret_cast<int*>(reinterpret_cast<long long*>(base + 32) + S::kEnt) + g * S::kHdr;
   for (int i = lane; i < S::kPhys; i += 32) bm[i] = 0u;
   sm[lane] = 0u;
   __syncwarp();
@@ -584,32 +590,40 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 8) bmr_group_symbolic_kernel
 // step the lanes of a group write distinct slots: plain shared-memory adds, no
 // atomics (a Laplacian row repeats 12 of its 25 product columns).
 template <typename T, int G>
-constexpr size_t grp_numeric_warp_bytes() {
+struct GrpNumLayout {
   using S = GrpShape<G>;
-  return static_cast<size_t>(S::kRows) * kBmrMaxA * G * (4 + sizeof(T)) +
-         static_cast<size_t>(S::kEnt) * (sizeof(long long) + sizeof(T) + sizeof(int));
+  static constexpr int kValStride = S::kCap + S::kPadBytes / static_cast<int>(sizeof(T));
+  static constexpr int kKeyStride = S::kCap + S::kPadBytes / 4;
+  static constexpr size_t kKeyOff = static_cast<size_t>(S::kRows) * kValStride * sizeof(T);
+  static constexpr size_t kB0Off = kKeyOff + static_cast<size_t>(S::kRows) * kKeyStride * 4;
+  static constexpr size_t kAOff = kB0Off + static_cast<size_t>(S::kEnt) * sizeof(long long);
+  static constexpr size_t kLenOff = kAOff + static_cast<size_t>(S::kEnt) * sizeof(T);
+  static constexpr size_t kBytes = kLenOff + static_cast<size_t>(S::kEnt) * sizeof(int);
+  static_assert(kB0Off % 8 == 0 && kAOff % sizeof(T) == 0 && kBytes % 8 == 0, "aligned arrays");
+};
+
+template <typename T, int G>
+constexpr size_t grp_numeric_warp_bytes() {
+  return GrpNumLayout<T, G>::kBytes;
 }
 
 template <typename T, int G>
 __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(const RowPlan<T> p) {
   using S = GrpShape<G>;
-  constexpr int kCap = kBmrMaxA * G;  // products (so entries) of a row at most
+  constexpr int kCap = S::kCap;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int sub = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int g = lane / G, gl = lane % G;
   // Per warp: staging values and columns of every group, then the stored A
   // entries of every group (B row start, A value, B row length).
+  using L = GrpNumLayout<T, G>;
   unsigned char* ws = smem_raw + static_cast<size_t>(sub) * grp_numeric_warp_bytes<T, G>();
-  constexpr size_t kKeyOff = static_cast<size_t>(S::kRows) * kCap * sizeof(T);
-  constexpr size_t kB0Off = kKeyOff + static_cast<size_t>(S::kRows) * kCap * 4;
-  constexpr size_t kAOff = kB0Off + static_cast<size_t>(S::kEnt) * sizeof(long long);
-  constexpr size_t kLenOff = kAOff + static_cast<size_t>(S::kEnt) * sizeof(T);
-  T* st_val = reinterpret_cast<T*>(ws) + g * kCap;
-  int* st_key = reinterpret_cast<int*>(ws + kKeyOff) + g * kCap;
-  long long* h_b0 = reinterpret_cast<long long*>(ws + kB0Off) + g * kBmrMaxA;
-  T* h_a = reinterpret_cast<T*>(ws + kAOff) + g * kBmrMaxA;
-  int* h_len = reinterpret_cast<int*>(ws + kLenOff) + g * kBmrMaxA;
+  T* st_val = reinterpret_cast<T*>(ws) + g * L::kValStride;
+  int* st_key = reinterpret_cast<int*>(ws + L::kKeyOff) + g * L::kKeyStride;
+  long long* h_b0 = reinterpret_cast<long long*>(ws + L::kB0Off) + g * S::kHdr;
+  T* h_a = reinterpret_cast<T*>(ws + L::kAOff) + g * S::kHdr;
+  int* h_len = reinterpret_cast<int*>(ws + L::kLenOff) + g * S::kHdr;
 
   const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
   for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * S::kRows; r0 < p.seg_len;
