@@ -713,16 +713,25 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(
 // kClsBmrWide, lo = 0); every other row goes to `pending` for the analysis
 // kernel.  Counts per class are added to the summary.
 //
-// One CTA of kPlanThreads threads (two warps) works on one row, so the
-// bitmap of a row is shared by all of them: thread t owns the contiguous
-// words [t * WPT, (t + 1) * WPT) (bits of columns [32 t WPT, 32 (t + 1) WPT)).
-// After the product bits are set, every thread counts the bits of its own
-// words in one sweep (no search for the non-zero words: the sweep is
-// branch-free and, with 32 words per thread, reads them as eight 16-byte
-// chunks), the CTA scans the counts, and every thread stores the rank of
-// the first column of each of its words.  A product's rank is then that word
-// rank plus the bits below it in its word.
+// One CTA of two warps works on one row at a time.  The products are split
+// by the steps of the one-warp numeric kernel (lane l, step s: element l % G
+// of the B row of stored A entry s * (32 / G) + l / G): warp w takes the
+// steps s = w, w + 2, ..., so every thread stores the ranks of products that
+// the same lane of the numeric kernel reads back.  The row's bitmap covers
+// all columns: thread t owns the contiguous words [t * WPT, (t + 1) * WPT)
+// (bits of columns [32 t WPT, 32 (t + 1) WPT)).  After the product bits are
+// set, every thread counts the bits of its own words in one branch-free
+// sweep of 16-byte chunks, each warp scans its counts, and every thread
+// stores the rank (within its warp's half of the columns) of the first
+// column of each of its words.  A product's rank is then that word rank,
+// plus warp 0's count for a column of warp 1's half, plus the bits below it
+// in its word; the sweep's chunk order clears the bitmap for the next row.
+//
+// Row headers (the B row extent of every stored A entry) are fetched for
+// kPlanHdrRows rows at a time.
 constexpr int kPlanThreads = 64;
+constexpr int kPlanHdrRows = 4;
+static_assert(kPlanHdrRows * kBmrMaxA == kPlanThreads, "one header entry per thread");
 // Sparsest row the planning pass takes: its sweep and clear cost the same for
 // every row of a launch (the whole bitmap), so rows with fewer products go to
 // the hash bins, whose cost follows the product count.  At 16 words per
@@ -731,238 +740,217 @@ constexpr long long kPlanWordsPerProduct = 16;
 
 template <int LOGW>
 struct PlanShape {
+  static_assert(LOGW >= 7 && LOGW <= 11, "two to thirty-two words per thread");
   static constexpr int kWords = 1 << LOGW;
-  static constexpr int kWPT = kWords >= kPlanThreads ? kWords / kPlanThreads : 1;  // words per thread
-  static constexpr int kPhysWords = kWPT * kPlanThreads;
-  // 32 words per thread: thread-major rows of eight 16-byte chunks, chunk c of
-  // thread t at position c ^ (t % 8), so the eight threads of a quarter warp
-  // read eight different bank groups.  Fewer: word i of thread t at i * 64 + t.
-  static constexpr bool kVec = kWPT == 32;
-  static constexpr size_t bytes() { return static_cast<size_t>(kPhysWords) * 6; }  // bitmap + uint16 word ranks
+  static constexpr int kWPT = kWords / kPlanThreads;  // words per thread
+  // bitmap, uint16 word ranks, per header entry {length, B position}, per header row {na, ub, taken}
+  static constexpr size_t kBytes = static_cast<size_t>(kWords) * 6 + kPlanThreads * 8 + kPlanHdrRows * 16;
 };
-static_assert(kPlanThreads == 64, "the shapes below assume 64 threads");
-// 16 CTAs per SM (the shared-memory limit): 64 registers a thread.
-constexpr int kPlanMinBlocks = 16;
 
+// Position of bitmap word w: for 32 words per thread (eight 16-byte chunks),
+// chunk c of thread t sits at t * 8 + (c ^ (t % 8)), so the eight threads of
+// a quarter warp that read their chunk c together hit eight different groups
+// of four banks; for 8 words per thread (two chunks) chunk c sits at
+// t * 2 + (c ^ ((t / 4) % 2)); for 2 words per thread, in order.
 template <class S>
-__device__ __forceinline__ uint32_t plan_phys(uint32_t w) {
-  if constexpr (S::kVec) {
-    // thread t = w / 32, word i = w % 32: chunk bits (2..4) of w XOR t % 8 (bits 5..7)
+__device__ __forceinline__ uint32_t plan_bm(uint32_t w) {
+  if constexpr (S::kWPT == 32) {
     return w ^ ((w >> 3) & 0x1cu);
+  } else if constexpr (S::kWPT == 8) {
+    return w ^ ((w >> 3) & 0x4u);
   } else {
-    return (w % S::kWPT) * kPlanThreads + w / S::kWPT;
+    return w;
   }
 }
-
-// Position of word w's rank in the uint16 rank array: for 32 words per thread,
-// thread-major rows of four 16-byte chunks (eight ranks each), chunk q of
-// thread t at position q ^ ((t / 2) % 4) (a conflict-free 16-byte store per
-// quarter warp); otherwise the bitmap's layout.
+// Position of word w's rank in the uint16 rank array: for 32 words per
+// thread (four chunks of eight ranks), chunk q of thread t at
+// t * 4 + (q ^ ((t / 2) % 4)); fewer words, in order (one 16-byte or 4-byte
+// store per thread).
 template <class S>
 __device__ __forceinline__ uint32_t plan_pre(uint32_t w) {
-  if constexpr (S::kVec) {
-    // chunk bits (3..4) of w XOR (t / 2) % 4 (bits 6..7)
+  if constexpr (S::kWPT == 32) {
     return w ^ ((w >> 3) & 0x18u);
   } else {
-    return plan_phys<S>(w);
+    return w;
   }
 }
 
 template <typename T, int LOGW, int G>
-__global__ void __launch_bounds__(kPlanThreads, kPlanMinBlocks) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
-                                                                int64_t ncols, int32_t* pending) {
+__global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
+                                                                    int64_t ncols, int32_t* pending) {
   using S = PlanShape<LOGW>;
-  constexpr int kGroups = kPlanThreads / G;   // A entries per step
-  constexpr int kSteps = (kBmrMaxA + kGroups - 1) / kGroups;  // steps covering kBmrMaxA entries
-  constexpr int kW = kPlanThreads / 32;
-  constexpr int kLoc = (S::kWPT + 1) / 2;
+  constexpr int kGroups = 32 / G;
+  constexpr int kSteps = kBmrMaxA / kGroups;  // steps of the one-warp numeric layout
+  constexpr int kHalf = kSteps / 2;          // steps q and q + kHalf share one rank word
+  constexpr int kMy = kSteps / 2;            // steps of this warp: s = 2 * st + warp
+  constexpr int kLenShift = 58;              // header entry: length in bits 58..63, B position below
+  constexpr unsigned long long kPosMask = (1ull << kLenShift) - 1;
+  static_assert(kSteps % 2 == 0, "two warps share the steps");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint32_t* bm = reinterpret_cast<uint32_t*>(smem_raw);
-  uint16_t* pre = reinterpret_cast<uint16_t*>(smem_raw + static_cast<size_t>(S::kPhysWords) * 4);
-  __shared__ long long s_b0[kBmrMaxA];
-  __shared__ int s_len[kBmrMaxA];
-  __shared__ int s_red[2 * kW];
-  const int t = threadIdx.x;
-  const int lane = t & 31, warp = t >> 5;
-  const int grp = t / G, gl = t % G;
-  for (int i = t; i < S::kPhysWords; i += kPlanThreads) bm[i] = 0u;
-  __syncthreads();
+  uint16_t* pre = reinterpret_cast<uint16_t*>(smem_raw + static_cast<size_t>(S::kWords) * 4);
+  unsigned long long* h_ent = reinterpret_cast<unsigned long long*>(smem_raw + static_cast<size_t>(S::kWords) * 6);
+  int4* h_row = reinterpret_cast<int4*>(h_ent + kPlanThreads);
+  __shared__ int s_cnt[2];
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int grp = lane / G, gl = lane % G;
+  for (int i = t; i < S::kWords / 4; i += kPlanThreads) reinterpret_cast<uint4*>(bm)[i] = make_uint4(0u, 0u, 0u, 0u);
   const long long words = (ncols + 31) >> 5;
   int taken = 0;
   unsigned long long prod = 0;
 
-  for (int64_t row = blockIdx.x; row < ap.m; row += gridDim.x) {
-    const int64_t ra = p.A.rowptr[row];
-    const int64_t na64 = p.A.rowptr[row + 1] - ra;
-    bool ok = na64 >= 2 && na64 <= ap.bmr_max_a;
-    const int na = static_cast<int>(ok ? na64 : 0);
-    if (ok) {
-      int my_len = 0;
-      if (t < na) {
-        const int k = p.A.colidx[ra + t];
-        const long long b0 = p.B.rowptr[k];
-        my_len = static_cast<int>(p.B.rowptr[k + 1] - b0);
-        s_b0[t] = b0;
-        s_len[t] = my_len;
+  for (int64_t r0 = static_cast<int64_t>(blockIdx.x) * kPlanHdrRows; r0 < ap.m;
+       r0 += static_cast<int64_t>(gridDim.x) * kPlanHdrRows) {
+    __syncthreads();  // previous batch done with the header arrays (and the first bitmap clear)
+    // Batch header: thread t reads stored A entry j = t % 16 of row r0 + t / 16
+    // and the extent of its B row (rows with more than bmr_max_a entries are not read).
+    {
+      const int i = t / kBmrMaxA, j = t % kBmrMaxA;
+      long long ra_l = 0;
+      int na_l = 0;
+      if (lane < 2 && r0 + 2 * warp + lane < ap.m) {  // lanes 0, 1: the two rows of this warp
+        const int64_t r = r0 + 2 * warp + lane;
+        ra_l = p.A.rowptr[r];
+        const long long n = p.A.rowptr[r + 1] - ra_l;
+        na_l = static_cast<int>(n < kBmrMaxA + 1 ? n : kBmrMaxA + 1);
       }
-      int ub = my_len, mx = my_len;
+      const long long ra = __shfl_sync(kFull, ra_l, lane / kBmrMaxA);
+      const int na = __shfl_sync(kFull, na_l, lane / kBmrMaxA);
+      long long b0 = 0;
+      int len = 0;
+      if (j < na && na <= ap.bmr_max_a) {
+        const int k = p.A.colidx[ra + j];
+        b0 = p.B.rowptr[k];
+        const long long n = p.B.rowptr[k + 1] - b0;
+        len = static_cast<int>(n < G + 1 ? n : G + 1);  // a longer B row only has to fail the fit test
+      }
+      h_ent[t] = (static_cast<unsigned long long>(len) << kLenShift) | static_cast<unsigned long long>(b0);
+      int ub = len, mx = len;
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
+      for (int o = kBmrMaxA / 2; o > 0; o >>= 1) {
         ub += __shfl_xor_sync(kFull, ub, o);
         mx = max(mx, __shfl_xor_sync(kFull, mx, o));
       }
-      if (lane == 0) {
-        s_red[warp] = ub;
-        s_red[kW + warp] = mx;
+      if (j == 0) {
+        const bool ok = na >= 2 && na <= ap.bmr_max_a && ub > 0 && mx <= G &&
+                        words <= kPlanWordsPerProduct * static_cast<long long>(ub) + 64;
+        h_row[i] = make_int4(na, ub, ok ? 1 : 0, 0);
+      }
+    }
+    __syncthreads();
+    const int nrows = static_cast<int>(ap.m - r0 < kPlanHdrRows ? ap.m - r0 : kPlanHdrRows);
+#pragma unroll 1
+    for (int i = 0; i < nrows; ++i) {
+      const int64_t row = r0 + i;
+      const int4 hr = h_row[i];
+      if (!hr.z) {
+        if (t == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
+        continue;
+      }
+      // Products of this thread: step st is numeric step s = 2 * st + warp.
+      int col[kMy];
+#pragma unroll
+      for (int st = 0; st < kMy; ++st) {
+        const unsigned long long h = h_ent[i * kBmrMaxA + (2 * st + warp) * kGroups + grp];
+        col[st] = gl < static_cast<int>(h >> kLenShift) ? p.B.colidx[(h & kPosMask) + gl] : -1;
+      }
+      if (i > 0) __syncthreads();  // the previous row's clear is complete
+      // Set the product bits; a product that finds its bit set repeats a column.
+      uint32_t dup = 0;
+#pragma unroll
+      for (int st = 0; st < kMy; ++st) {
+        if (col[st] >= 0) {
+          const uint32_t off = static_cast<uint32_t>(col[st]);
+          const uint32_t bit = 1u << (off & 31u);
+          if (atomicOr(bm + plan_bm<S>(off >> 5), bit) & bit) dup |= 1u << st;
+        }
       }
       __syncthreads();
-      ub = 0;
-      mx = 0;
+      // Sweep: local rank of the first column of each of this thread's words,
+      // two per register (word 2k low half, 2k + 1 high half).
+      uint32_t loc[(S::kWPT + 1) / 2];
+      uint32_t run = 0;
+      if constexpr (S::kWPT >= 4) {
+        const uint4* mine = reinterpret_cast<const uint4*>(bm) + t * (S::kWPT / 4);
 #pragma unroll
-      for (int w2 = 0; w2 < kW; ++w2) {
-        ub += s_red[w2];
-        mx = max(mx, s_red[kW + w2]);
+        for (int c = 0; c < S::kWPT / 4; ++c) {
+          const uint4 v = mine[S::kWPT == 32 ? (c ^ (t & 7)) : S::kWPT == 8 ? (c ^ ((t >> 2) & 1)) : c];
+          const uint32_t r1 = run + __popc(v.x);
+          const uint32_t r2 = r1 + __popc(v.y);
+          const uint32_t r3 = r2 + __popc(v.z);
+          loc[2 * c] = run | (r1 << 16);
+          loc[2 * c + 1] = r2 | (r3 << 16);
+          run = r3 + __popc(v.w);
+        }
+      } else {
+        const uint2 v = reinterpret_cast<const uint2*>(bm)[t];
+        loc[0] = __popc(v.x) << 16;
+        run = __popc(v.x) + __popc(v.y);
       }
-      ok = ub > 0 && mx <= G && words <= kPlanWordsPerProduct * static_cast<long long>(ub) + 64;
-      if (ok) {
-        // products of this thread: step s covers A entry j = s * kGroups + grp
-        int col[kSteps];
+      uint32_t incl = run;
 #pragma unroll
-        for (int st = 0; st < kSteps; ++st) {
-          const int j = st * kGroups + grp;
-          col[st] = -1;
-          if (j < na && gl < s_len[j]) col[st] = p.B.colidx[s_b0[j] + gl];
-        }
-        uint32_t dup = 0;
-#pragma unroll
-        for (int st = 0; st < kSteps; ++st) {
-          if (col[st] >= 0) {
-            const uint32_t off = static_cast<uint32_t>(col[st]);
-            const uint32_t bit = 1u << (off & 31u);
-            if (atomicOr(bm + plan_phys<S>(off >> 5), bit) & bit) dup |= 1u << st;
-          }
-        }
-        __syncthreads();
-        // Sweep: local rank of the first column of each of this thread's words,
-        // two per register (word 2k low half, 2k + 1 high half).
-        uint32_t loc[kLoc];
-        int run = 0;
-        if constexpr (S::kVec) {
-          const uint4* mine = reinterpret_cast<const uint4*>(bm + t * 32);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint4 v = mine[c ^ (t & 7)];
-            loc[2 * c] = static_cast<uint32_t>(run);
-            run += __popc(v.x);
-            loc[2 * c] |= static_cast<uint32_t>(run) << 16;
-            run += __popc(v.y);
-            loc[2 * c + 1] = static_cast<uint32_t>(run);
-            run += __popc(v.z);
-            loc[2 * c + 1] |= static_cast<uint32_t>(run) << 16;
-            run += __popc(v.w);
-          }
-        } else {
-#pragma unroll
-          for (int i = 0; i < S::kWPT; ++i) {
-            const int pc = __popc(bm[i * kPlanThreads + t]);
-            if (i & 1) {
-              loc[i >> 1] |= static_cast<uint32_t>(run) << 16;
-            } else {
-              loc[i >> 1] = static_cast<uint32_t>(run);
-            }
-            run += pc;
-          }
-        }
-        // Exclusive scan of the per-thread counts in thread order (= column order).
-        int incl = run;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_up_sync(kFull, incl, o);
-          if (lane >= o) incl += y;
-        }
-        if (lane == 31) s_red[warp] = incl;
-        __syncthreads();
-        int before = 0, total = 0;
-#pragma unroll
-        for (int w2 = 0; w2 < kW; ++w2) {
-          const int v = s_red[w2];
-          before += w2 < warp ? v : 0;
-          total += v;
-        }
-        // Word ranks = thread base + local ranks (both halves: no carry, every rank <= kBmrCap).
-        const uint32_t base = static_cast<uint32_t>(before + incl - run);
-        const uint32_t base2 = base | (base << 16);
-        if constexpr (S::kVec) {
-          uint4* mine = reinterpret_cast<uint4*>(pre + t * 32);
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            mine[q ^ ((t >> 1) & 3)] =
-                make_uint4(loc[4 * q] + base2, loc[4 * q + 1] + base2, loc[4 * q + 2] + base2, loc[4 * q + 3] + base2);
-        } else {
-#pragma unroll
-          for (int i = 0; i < S::kWPT; ++i)
-            pre[i * kPlanThreads + t] = static_cast<uint16_t>(((loc[i >> 1] >> (16 * (i & 1))) & 0xffffu) + base);
-        }
-        __syncthreads();
-        int rk[kSteps];
-#pragma unroll
-        for (int st = 0; st < kSteps; ++st) {
-          rk[st] = 0;
-          if (col[st] >= 0) {
-            const uint32_t off = static_cast<uint32_t>(col[st]);
-            const uint32_t w = off >> 5;
-            rk[st] = (pre[plan_pre<S>(w)] + __popc(bm[plan_phys<S>(w)] & ((1u << (off & 31u)) - 1u))) |
-                     static_cast<int>(((dup >> st) & 1u) << 15);
-          }
-        }
-        // Stored A entry j of this thread at step st is j = st * kGroups + grp;
-        // in the one-warp numeric kernel it sits at step j / kNumGroups of
-        // lane (j % kNumGroups) * G + gl.
-        constexpr int kNumGroups = 32 / G;
-        constexpr int kNumSteps = kBmrMaxA / kNumGroups;
-        if constexpr (8 % kGroups == 0) {
-          // entries j and j + 8 (steps st and st + kPair) share one rank word
-          constexpr int kPair = 8 / kGroups;
-          uint32_t* ranks32 = reinterpret_cast<uint32_t*>(p.ranks + row * kBmrSlots);
-#pragma unroll
-          for (int st = 0; st < kPair; ++st) {
-            const int j = st * kGroups + grp;
-            if (col[st] >= 0 || col[st + kPair] >= 0)
-              ranks32[rank_word<kNumSteps>(j / kNumGroups, (j % kNumGroups) * G + gl)] = rank_pack(rk[st], rk[st + kPair]);
-          }
-        } else {
-          uint16_t* ranks = p.ranks + row * kBmrSlots;
-#pragma unroll
-          for (int st = 0; st < kSteps; ++st) {
-            const int j = st * kGroups + grp;
-            const int sn = j / kNumGroups;
-            if (col[st] >= 0)
-              ranks[2 * rank_word<kNumSteps>(sn, (j % kNumGroups) * G + gl) + (sn >= kNumSteps / 2)] =
-                  static_cast<uint16_t>(rk[st]);
-          }
-        }
-        __syncthreads();
-        // Clear this thread's words (conflict-free).
-        if constexpr (S::kVec) {
-          uint4* mine = reinterpret_cast<uint4*>(bm + t * 32);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) mine[c ^ (t & 7)] = make_uint4(0u, 0u, 0u, 0u);  // same order as the sweep
-        } else {
-#pragma unroll
-          for (int i = 0; i < S::kWPT; ++i) bm[i * kPlanThreads + t] = 0u;
-        }
-        if (t == 0) {
-          p.c_rowptr[row + 1] = total;
-          p.cls[row] = kClsBmrWide;
-          p.lo[row] = 0;
-          p.hi[row] = static_cast<int32_t>(ncols - 1);
-          ++taken;
-          prod += static_cast<unsigned long long>(ub);
-        }
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
       }
-      __syncthreads();  // bitmap clear and s_b0/s_len reuse
+      if (lane == 31) s_cnt[warp] = static_cast<int>(incl);
+      // Word ranks within this warp's half (both halves of a register: no carry, every rank <= kBmrCap).
+      const uint32_t base = incl - run;
+      const uint32_t base2 = base | (base << 16);
+      if constexpr (S::kWPT == 32) {
+        uint4* pm = reinterpret_cast<uint4*>(pre) + t * 4;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          pm[q ^ ((t >> 1) & 3)] = make_uint4(loc[4 * q] + base2, loc[4 * q + 1] + base2, loc[4 * q + 2] + base2,
+                                              loc[4 * q + 3] + base2);
+      } else if constexpr (S::kWPT == 8) {
+        reinterpret_cast<uint4*>(pre)[t] = make_uint4(loc[0] + base2, loc[1] + base2, loc[2] + base2, loc[3] + base2);
+      } else {
+        reinterpret_cast<uint32_t*>(pre)[t] = loc[0] + base2;
+      }
+      __syncthreads();
+      const uint32_t lower = static_cast<uint32_t>(s_cnt[0]);  // entries in warp 0's half of the columns
+      // Rank of this thread's step st product: its word's rank within its
+      // half, warp 0's count for a column of warp 1's half, and the bits below
+      // it in its word.
+      auto rank_of = [&](int st) -> uint32_t {
+        if (col[st] < 0) return 0u;
+        const uint32_t off = static_cast<uint32_t>(col[st]);
+        const uint32_t w = off >> 5;
+        const uint32_t half = (w >> (LOGW - 1)) & 1u;
+        return (pre[plan_pre<S>(w)] + (half ? lower : 0u) +
+                __popc(bm[plan_bm<S>(w)] & ((1u << (off & 31u)) - 1u))) |
+               ((dup << (15 - st)) & 0x8000u);
+      };
+      uint32_t* ranks32 = reinterpret_cast<uint32_t*>(p.ranks + row * kBmrSlots);
+      if constexpr (kHalf % 2 == 0) {
+        // numeric steps s and s + kHalf (st and st + kHalf / 2 here) share a rank word
+#pragma unroll
+        for (int st = 0; st < kHalf / 2; ++st)
+          ranks32[((2 * st + warp) << 5) | lane] = rank_of(st) | (rank_of(st + kHalf / 2) << 16);
+      } else {
+        // one step per warp (G = 4): warp w fills half w of rank word 0
+        p.ranks[row * kBmrSlots + 2 * lane + warp] = static_cast<uint16_t>(rank_of(0));
+      }
+      __syncthreads();
+      // Clear this thread's words (conflict-free, the sweep's order).
+      if constexpr (S::kWPT >= 4) {
+        uint4* mine = reinterpret_cast<uint4*>(bm) + t * (S::kWPT / 4);
+#pragma unroll
+        for (int c = 0; c < S::kWPT / 4; ++c)
+          mine[S::kWPT == 32 ? (c ^ (t & 7)) : S::kWPT == 8 ? (c ^ ((t >> 2) & 1)) : c] = make_uint4(0u, 0u, 0u, 0u);
+      } else {
+        reinterpret_cast<uint2*>(bm)[t] = make_uint2(0u, 0u);
+      }
+      if (t == 0) {
+        p.c_rowptr[row + 1] = s_cnt[0] + s_cnt[1];
+        p.cls[row] = kClsBmrWide;
+        p.lo[row] = 0;
+        p.hi[row] = static_cast<int32_t>(ncols - 1);
+      }
+      ++taken;
+      prod += static_cast<unsigned long long>(hr.y);
     }
-    if (!ok && t == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
   }
   if (t == 0) {
     if (taken) atomicAdd(&p.sum->seg_count[kSegBmrWide], taken);
@@ -1023,10 +1011,11 @@ void launch_bmr_w(const RowPlan<T>& p, bool numeric, int num_sms, cudaStream_t s
 template <typename T, int LOGW, int G>
 void launch_plan_g(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, int32_t* pending, int num_sms,
                    cudaStream_t s) {
-  const size_t smem = PlanShape<LOGW>::bytes();
+  const size_t smem = PlanShape<LOGW>::kBytes;
   static int per_sm = 0;
   if (per_sm == 0) per_sm = occupancy(bmr_plan_kernel<T, LOGW, G>, kPlanThreads, smem);
-  const int64_t grid = clamp_grid(ap.m, num_sms, per_sm);
+  constexpr int64_t kPerCta = kPlanHdrRows;
+  const int64_t grid = clamp_grid((ap.m + kPerCta - 1) / kPerCta, num_sms, per_sm);
   bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), kPlanThreads, smem, s>>>(p, ap, ncols, pending);
 }
 
