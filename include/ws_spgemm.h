@@ -298,8 +298,10 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
  *   key 1: largest product count of a row that uses the shared-memory hash
  *          path (default 4096; smaller values send more rows to the
  *          dense-window path, 0 sends every multi-entry row there)
- *   key 2: longest run of occupied hash slots the sort-free ranking accepts
- *          (default 64; smaller values send more rows to the sorting path)
+ *   key 2: longest run of occupied slots a row's hash table may hold
+ *          (default 64; a row with a longer run, or whose probes wrap
+ *          around the table, uses the sorting path; smaller values send
+ *          more rows there)
  *   key 3: dense-window slice width in columns (default 8192 for double,
  *          16384 for float; must be a multiple of 1024, 0 = default)
  *   key 4: widest column range of a row that uses the bitmap path

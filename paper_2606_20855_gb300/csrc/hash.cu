@@ -11,23 +11,28 @@
 // Monotone hash.  Every product column of the row lies in [lo, hi] (B's rows
 // are sorted).  The home slot of column c is
 //     h(c) = floor((c - lo) * T / span),  span = hi - lo + 1,
-// (h(c) = c - lo when span <= T), which never decreases as c grows.  With
-// linear probing and no wrap-around, every key's home lies inside the run of
-// occupied slots ("cluster") that holds the key, so keys of an earlier
-// cluster are smaller than keys of a later one.  Hence the sorted position of
-// the key in slot s is
-//     (#occupied slots before s) - (s - cluster_start) + #{keys of s's cluster < key(s)}
-// and the row is written in sorted column order without a sort.  The
-// symbolic pass checks each row's table for a wrap-around or a cluster longer
-// than the ranking limit and re-routes such rows to the sorting path.  The
-// set of occupied slots of a linear-probing table does not depend on the
-// insertion order, so the numeric pass (same keys, same table, same hash)
-// sees exactly the clusters the symbolic pass checked.
-//
+// (h(c) = c - lo when span <= T), which never decreases as c grows.
+// Symbolic pass: plain linear probing counts the distinct columns.  The set
+// of occupied slots of a linear-probing table depends only on the keys'
+// home slots, not on the insertion order or on which key of a run sits
+// where, so the pass also checks the run structure the numeric pass will
+// meet: a row whose probes wrap around the table (or, as a tuning limit,
+// whose table holds a long run) is re-routed to the sorting path.
+// Numeric pass: ordered linear probing -- an inserted key moves on past
+// smaller keys and takes the place of the first larger one, which then moves
+// on in its turn (a compare-and-swap per exchange, no wrap-around).  Keys
+// only move forward and a slot's key only ever shrinks, so every run of
+// occupied slots ends sorted and, with the monotone hash, so does the whole
+// table: the output position of the key in slot s is the number of occupied
+// slots before s, and the row is written in column order without a sort.
+// Once every key is in place, each product finds its key's slot and adds
+// its value there.
 // Table sizes: bin b holds rows with at most 32 << b products whose home
 // slots span 64 << b slots, so the load factor is at most 1/2.  The table
 // has tail_slots() extra slots past the home range, so a run of keys that reaches
 // the end of the home range continues upward instead of wrapping to slot 0.
+#include <type_traits>
+
 #include "ws_internal.cuh"
 
 namespace wsk {
@@ -82,6 +87,37 @@ __device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint
     }
   }
   return kInsFailed | wrapped;
+}
+
+// Ordered insert of key c (numeric pass): returns kInsNew if the insert
+// filled an empty slot (one more distinct key in the table), 0 if the key
+// (or a key it displaced) met an equal key, kInsFailed if a key would move
+// past the last slot.  Keys of a run stay sorted; no wrap-around.
+__device__ __forceinline__ int ordered_insert(int* keys, uint32_t h, uint32_t nslots, int c) {
+  volatile int* vk = keys;
+  // Every retry follows a successful change of the slot by another insert,
+  // and a slot changes at most once per key of the row; the guard only bounds
+  // the loop for a broken table.
+  for (uint32_t guard = 0; h < nslots && guard < 8u * nslots; ++guard) {
+    const int cur = vk[h];
+    if (cur == kEmptyKey || cur > c) {
+      const int old = atomicCAS(&keys[h], cur, c);
+      if (old != cur) continue;       // the slot changed: look again
+      if (cur == kEmptyKey) return kInsNew;
+      c = cur;                        // carry the displaced larger key on
+    } else if (cur == c) {
+      return 0;
+    }
+    ++h;
+  }
+  return kInsFailed;
+}
+
+// Slot of key c in a finished ordered table (every slot from its home slot
+// up to it is occupied); nslots if it is missing.
+__device__ __forceinline__ uint32_t find_key(const int* keys, uint32_t h, uint32_t nslots, int c) {
+  while (h < nslots && keys[h] != c) ++h;
+  return h;
 }
 
 // True if the table holds a run of more than `limit` occupied slots.  Called
@@ -168,65 +204,84 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
     // Accumulate: w[j] += A[i,k] * B[k,j] for every stored A[i,k], B[k,j].
     // The team first stages a chunk of the row's A entries (B-row bounds and
     // A values) in shared memory, then every group of gsize lanes walks B
-    // rows, loading kUnroll B entries before it inserts any of them.
+    // rows, loading kUnroll B entries before it handles any of them.
+    // Symbolic pass: one walk, plain probing.  Numeric pass: a walk that
+    // places the keys (ordered probing), then a walk that adds the values.
     int my_new = 0, my_flags = 0;
-#define WS_INSERT(c_, v_)                                                                                     \
-  do {                                                                                                        \
-    const uint32_t d_ = static_cast<uint32_t>((c_) - lo);                                                     \
-    const uint32_t h_ = ident ? d_ : static_cast<uint32_t>((static_cast<unsigned long long>(d_) * mul) >> 32); \
-    const int r_ = probe_insert<NUMERIC>(keys, vals, h_, kS, (c_), (v_));                                     \
-    my_new += r_ & kInsNew;                                                                                   \
-    my_flags |= r_;                                                                                           \
-  } while (0)
     long long* st_b0 = s_b0 + sub * kNT;
     long long* st_b1 = s_b1 + sub * kNT;
     T* st_a = s_a + sub * kNT;
     const int64_t ra = p.A.rowptr[row], re = p.A.rowptr[row + 1];
-    for (int64_t cb = ra; cb < re; cb += kNT) {
-      const int n = static_cast<int>(min(static_cast<int64_t>(kNT), re - cb));
-      if (t < n) {
-        const int k = p.A.colidx[cb + t];
-        st_b0[t] = p.B.rowptr[k];
-        st_b1[t] = p.B.rowptr[k + 1];
-        if constexpr (NUMERIC) st_a[t] = p.A.vals[cb + t];
-      }
-      team_sync<WPR>();
-      for (int j0 = grp; j0 < n; j0 += ngrp * kUnroll) {
-        int cc[kUnroll];
-        T vv[kUnroll];
+    auto home = [&](int c) -> uint32_t {
+      const uint32_t d = static_cast<uint32_t>(c - lo);
+      return ident ? d : static_cast<uint32_t>((static_cast<unsigned long long>(d) * mul) >> 32);
+    };
+    // Calls f(column, scaled value) for every product of the row this lane
+    // owns (with_vals false: the value is not loaded and f gets 0).
+    auto for_products = [&](auto with_vals, auto&& f) {
+      constexpr bool kVals = NUMERIC && decltype(with_vals)::value;
+      for (int64_t cb = ra; cb < re; cb += kNT) {
+        const int n = static_cast<int>(min(static_cast<int64_t>(kNT), re - cb));
+        if (t < n) {
+          const int k = p.A.colidx[cb + t];
+          st_b0[t] = p.B.rowptr[k];
+          st_b1[t] = p.B.rowptr[k + 1];
+          if constexpr (kVals) st_a[t] = p.A.vals[cb + t];
+        }
+        team_sync<WPR>();
+        for (int j0 = grp; j0 < n; j0 += ngrp * kUnroll) {
+          int cc[kUnroll];
+          T vv[kUnroll];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-          const int j = j0 + u * ngrp;
-          cc[u] = -1;
-          vv[u] = T(0);
-          if (j < n) {
-            const long long q = st_b0[j] + gl;
-            if (q < st_b1[j]) {
-              cc[u] = p.B.colidx[q];
-              if constexpr (NUMERIC) vv[u] = st_a[j] * p.B.vals[q];
+          for (int u = 0; u < kUnroll; ++u) {
+            const int j = j0 + u * ngrp;
+            cc[u] = -1;
+            vv[u] = T(0);
+            if (j < n) {
+              const long long q = st_b0[j] + gl;
+              if (q < st_b1[j]) {
+                cc[u] = p.B.colidx[q];
+                if constexpr (kVals) vv[u] = st_a[j] * p.B.vals[q];
+              }
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < kUnroll; ++u) {
+            if (cc[u] >= 0) f(cc[u], vv[u]);
+          }
+          // B rows longer than the group: the rest of each row.
+#pragma unroll 1
+          for (int u = 0; u < kUnroll; ++u) {
+            const int j = j0 + u * ngrp;
+            if (j >= n) break;
+            const long long qe = st_b1[j];
+            for (long long q = st_b0[j] + gl + gsize; q < qe; q += gsize) {
+              T v = T(0);
+              if constexpr (kVals) v = st_a[j] * p.B.vals[q];
+              f(p.B.colidx[q], v);
             }
           }
         }
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-          if (cc[u] >= 0) WS_INSERT(cc[u], vv[u]);
-        }
-        // B rows longer than the group: the rest of each row.
-#pragma unroll 1
-        for (int u = 0; u < kUnroll; ++u) {
-          const int j = j0 + u * ngrp;
-          if (j >= n) break;
-          const long long qe = st_b1[j];
-          for (long long q = st_b0[j] + gl + gsize; q < qe; q += gsize) {
-            T v = T(0);
-            if constexpr (NUMERIC) v = st_a[j] * p.B.vals[q];
-            WS_INSERT(p.B.colidx[q], v);
-          }
-        }
+        team_sync<WPR>();
       }
-      team_sync<WPR>();
+    };
+    if constexpr (!NUMERIC) {
+      for_products(std::false_type{}, [&](int c, T) {
+        const int r = probe_insert<false>(keys, vals, home(c), kS, c, T(0));
+        my_new += r & kInsNew;
+        my_flags |= r;
+      });
+    } else {
+      for_products(std::false_type{}, [&](int c, T) { my_flags |= ordered_insert(keys, home(c), kS, c); });
+      for_products(std::true_type{}, [&](int c, T v) {
+        const uint32_t h = find_key(keys, home(c), kS, c);
+        if (h < static_cast<uint32_t>(kS)) {
+          atomic_add_value(&vals[h], v);
+        } else {
+          my_flags |= kInsFailed;
+        }
+      });
     }
-#undef WS_INSERT
     const bool wrapped = (my_flags & kInsWrapped) != 0;
     const bool failed = (my_flags & kInsFailed) != 0;
 
@@ -278,35 +333,16 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
       }
       const int64_t base = p.c_rowptr[row];
       const int64_t cnt = p.c_rowptr[row + 1] - base;
-      const int limit = p.run_limit;
-      bool rank_err = false, count_err = false;
+      bool count_err = false;
       for (int c0 = s_begin; c0 < s_begin + kPerWarp; c0 += 32) {
         const int s = c0 + lane;
         const int key = keys[s];
         const bool occ = key != kEmptyKey;
         const unsigned m = __ballot_sync(kFull, occ);
         if (occ) {
-          const int before = carry + __popc(m & ((1u << lane) - 1u));
-          int rk = 0;
-          int cs = s;
-          int steps = 0;
-          while (cs > 0 && steps < limit) {
-            const int kk = keys[cs - 1];
-            if (kk == kEmptyKey) break;
-            rk += kk < key;
-            --cs;
-            ++steps;
-          }
-          if (cs > 0 && steps == limit && keys[cs - 1] != kEmptyKey) rank_err = true;
-          int u = s + 1;
-          for (steps = 0; u < kS && steps < limit; ++u, ++steps) {
-            const int kk = keys[u];
-            if (kk == kEmptyKey) break;
-            rk += kk < key;
-          }
-          if (u < kS && steps == limit && keys[u] != kEmptyKey) rank_err = true;
-          const int64_t pos = static_cast<int64_t>(before) - (s - cs) + rk;
-          if (pos >= 0 && pos < cnt) {
+          // The table is sorted: the key's position is the count of occupied slots before it.
+          const int64_t pos = static_cast<int64_t>(carry) + __popc(m & ((1u << lane) - 1u));
+          if (pos < cnt) {
             p.c_colidx[base + pos] = key;
             p.c_vals[base + pos] = vals[s];
           } else {
@@ -318,7 +354,6 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
       if (WPR == 1 || warp == WPR - 1) {
         if (carry != cnt) count_err = true;
       }
-      if (__any_sync(kFull, rank_err) && lane == 0) atomicOr(&p.sum->status, kErrRank);
       if (__any_sync(kFull, count_err) && lane == 0) atomicOr(&p.sum->status, kErrCount);
       if (__any_sync(kFull, failed) && lane == 0) atomicOr(&p.sum->status, kErrProbe);
       team_sync<WPR>();

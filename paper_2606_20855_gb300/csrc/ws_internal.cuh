@@ -160,7 +160,7 @@ struct RowPlan {
   int64_t seg_begin;   // first position in perm of the segment a kernel processes
   int64_t seg_len;     // rows in that segment
   int log2_group;      // lanes per stored A entry when walking B rows (1 << log2_group)
-  int run_limit;       // longest occupied run the sort-free ranking accepts
+  int run_limit;       // longest occupied run a hash row may hold (longer: sorting path)
   int dense_width;     // dense-window slice width in columns
 };
 
