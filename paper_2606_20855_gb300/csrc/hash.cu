@@ -55,32 +55,20 @@ __device__ __forceinline__ void team_sync() {
   }
 }
 
-template <typename T>
-__device__ __forceinline__ void atomic_add_value(T* addr, T v) {
-  atomicAdd(addr, v);
-}
-
-// Inserts key c (and adds v when NUMERIC) into the table.  Returns a bit set:
+// Inserts key c into the symbolic pass's key table.  Returns a bit set:
 // kInsNew if the key was new, kInsWrapped if the probe wrapped from the last
 // slot to slot 0, kInsFailed if every slot was probed.
 constexpr int kInsNew = 1, kInsWrapped = 2, kInsFailed = 4;
-template <bool NUMERIC, typename T>
-__device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint32_t nslots, int c, T v) {
+__device__ __forceinline__ int probe_insert(int* keys, uint32_t h, uint32_t nslots, int c) {
   volatile int* vk = keys;
   int wrapped = 0;
   for (uint32_t n = 0; n < nslots; ++n) {
     int cur = vk[h];
     if (cur == kEmptyKey) {
       cur = atomicCAS(&keys[h], kEmptyKey, c);
-      if (cur == kEmptyKey) {
-        if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
-        return kInsNew | wrapped;
-      }
+      if (cur == kEmptyKey) return kInsNew | wrapped;
     }
-    if (cur == c) {
-      if constexpr (NUMERIC) atomic_add_value(&vals[h], v);
-      return wrapped;
-    }
+    if (cur == c) return wrapped;
     if (++h == nslots) {
       h = 0;
       wrapped = kInsWrapped;
@@ -89,35 +77,68 @@ __device__ __forceinline__ int probe_insert(int* keys, T* vals, uint32_t h, uint
   return kInsFailed | wrapped;
 }
 
-// Ordered insert of key c (numeric pass): returns kInsNew if the insert
-// filled an empty slot (one more distinct key in the table), 0 if the key
-// (or a key it displaced) met an equal key, kInsFailed if a key would move
-// past the last slot.  Keys of a run stay sorted; no wrap-around.
-__device__ __forceinline__ int ordered_insert(int* keys, uint32_t h, uint32_t nslots, int c) {
-  volatile int* vk = keys;
-  // Every retry follows a successful change of the slot by another insert,
-  // and a slot changes at most once per key of the row; the guard only bounds
-  // the loop for a broken table.
-  for (uint32_t guard = 0; h < nslots && guard < 8u * nslots; ++guard) {
-    const int cur = vk[h];
-    if (cur == kEmptyKey || cur > c) {
-      const int old = atomicCAS(&keys[h], cur, c);
-      if (old != cur) continue;       // the slot changed: look again
-      if (cur == kEmptyKey) return kInsNew;
-      c = cur;                        // carry the displaced larger key on
-    } else if (cur == c) {
-      return 0;
+// Numeric-pass slot: a column and its accumulated value in one word that a
+// single compare-and-swap replaces (8 bytes for float, 16 for double).  The
+// key sits in the low 32 bits; an empty slot has key -1 and value 0.
+template <typename T>
+struct PairSlot;
+template <>
+struct PairSlot<float> {
+  using W = unsigned long long;
+  static __device__ __forceinline__ W make(int c, float v) {
+    return static_cast<W>(static_cast<uint32_t>(c)) | (static_cast<W>(__float_as_uint(v)) << 32);
+  }
+  static __device__ __forceinline__ int key(W w) { return static_cast<int>(static_cast<uint32_t>(w)); }
+  static __device__ __forceinline__ float val(W w) { return __uint_as_float(static_cast<uint32_t>(w >> 32)); }
+};
+template <>
+struct PairSlot<double> {
+  using W = unsigned __int128;
+  static __device__ __forceinline__ W make(int c, double v) {
+    return static_cast<W>(static_cast<uint32_t>(c)) |
+           (static_cast<W>(static_cast<unsigned long long>(__double_as_longlong(v))) << 64);
+  }
+  static __device__ __forceinline__ int key(W w) { return static_cast<int>(static_cast<uint32_t>(w)); }
+  static __device__ __forceinline__ double val(W w) {
+    return __longlong_as_double(static_cast<long long>(static_cast<unsigned long long>(w >> 64)));
+  }
+};
+
+// Ordered insert of product (c, v) into the numeric pass's pair table:
+// returns 0, or kInsFailed if a pair would move past the last slot.  The
+// pair moves on past smaller keys; at the first larger key it takes that
+// slot and carries the displaced pair (key and value together) on; at an
+// empty slot it settles; at an equal key it adds its value there.  A slot's
+// key only ever shrinks and keys only move forward, so every run of
+// occupied slots stays sorted and no value is lost: a pair is either in the
+// table or carried by exactly one thread, and a carried pair that meets its
+// own key merges into it.  No wrap-around.
+template <typename T>
+__device__ __forceinline__ int ordered_insert_pair(typename PairSlot<T>::W* slots, uint32_t h, uint32_t nslots, int c, T v) {
+  using P = PairSlot<T>;
+  using W = typename P::W;
+  W carry = P::make(c, v);
+  // Every failed compare-and-swap follows a successful change of the slot by
+  // another insert; the guard only bounds the loop for a broken table.
+  for (uint32_t guard = 0; h < nslots && guard < 16u * nslots; ++guard) {
+    const W cur = slots[h];
+    const int kc = P::key(cur);
+    const int kn = P::key(carry);
+    W next;
+    if (kc == kEmptyKey || kc > kn) {
+      next = carry;
+    } else if (kc == kn) {
+      next = P::make(kn, P::val(cur) + P::val(carry));
+    } else {
+      ++h;
+      continue;
     }
+    if (atomicCAS(slots + h, cur, next) != cur) continue;  // the slot changed: look again
+    if (kc == kEmptyKey || kc == kn) return 0;
+    carry = cur;  // carry the displaced larger pair on
     ++h;
   }
   return kInsFailed;
-}
-
-// Slot of key c in a finished ordered table (every slot from its home slot
-// up to it is occupied); nslots if it is missing.
-__device__ __forceinline__ uint32_t find_key(const int* keys, uint32_t h, uint32_t nslots, int c) {
-  while (h < nslots && keys[h] != c) ++h;
-  return h;
 }
 
 // True if the table holds a run of more than `limit` occupied slots.  Called
@@ -143,12 +164,6 @@ __device__ __forceinline__ bool has_long_run(const int* keys, int nslots, int li
   return bad;
 }
 
-template <typename T>
-__device__ __forceinline__ void clear_values(T* vals, int n, int t, int nt) {
-  int4* v4 = reinterpret_cast<int4*>(vals);
-  const int n4 = static_cast<int>(n * sizeof(T) / sizeof(int4));
-  for (int s = t; s < n4; s += nt) v4[s] = make_int4(0, 0, 0, 0);
-}
 
 // LOGT: log2 of table slots; WPR: warps per row team; RPC: row teams per CTA.
 // The launch bounds let the compiler use up to 64 registers per thread.
@@ -168,9 +183,10 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
   const int t = threadIdx.x % kNT;
   const int lane = threadIdx.x & 31;
   const int warp = t >> 5;
+  using PW = typename PairSlot<T>::W;
+  // symbolic pass: keys; numeric pass: (key, value) pairs
   int* keys = reinterpret_cast<int*>(smem_raw) + sub * kS;
-  T* vals = nullptr;
-  if constexpr (NUMERIC) vals = reinterpret_cast<T*>(reinterpret_cast<int*>(smem_raw) + RPC * kS) + sub * kS;
+  PW* pairs = reinterpret_cast<PW*>(smem_raw) + sub * kS;
 
   const int lg = p.log2_group;
   const int gsize = 1 << lg;
@@ -191,9 +207,13 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
 
     // Clear the workspace (w .= 0).
     {
-      int4* k4 = reinterpret_cast<int4*>(keys);
-      for (int s = t; s < kS / 4; s += kNT) k4[s] = make_int4(kEmptyKey, kEmptyKey, kEmptyKey, kEmptyKey);
-      if constexpr (NUMERIC) clear_values(vals, kS, t, kNT);
+      if constexpr (NUMERIC) {
+        const PW empty = PairSlot<T>::make(kEmptyKey, T(0));
+        for (int s = t; s < kS; s += kNT) pairs[s] = empty;
+      } else {
+        int4* k4 = reinterpret_cast<int4*>(keys);
+        for (int s = t; s < kS / 4; s += kNT) k4[s] = make_int4(kEmptyKey, kEmptyKey, kEmptyKey, kEmptyKey);
+      }
       if constexpr (WPR > 1) {
         if (t < WPR) s_warp[t] = 0;
         if (t == 0) s_flags = 0;
@@ -267,20 +287,12 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
     };
     if constexpr (!NUMERIC) {
       for_products(std::false_type{}, [&](int c, T) {
-        const int r = probe_insert<false>(keys, vals, home(c), kS, c, T(0));
+        const int r = probe_insert(keys, home(c), kS, c);
         my_new += r & kInsNew;
         my_flags |= r;
       });
     } else {
-      for_products(std::false_type{}, [&](int c, T) { my_flags |= ordered_insert(keys, home(c), kS, c); });
-      for_products(std::true_type{}, [&](int c, T v) {
-        const uint32_t h = find_key(keys, home(c), kS, c);
-        if (h < static_cast<uint32_t>(kS)) {
-          atomic_add_value(&vals[h], v);
-        } else {
-          my_flags |= kInsFailed;
-        }
-      });
+      for_products(std::true_type{}, [&](int c, T v) { my_flags |= ordered_insert_pair<T>(pairs, home(c), kS, c, v); });
     }
     const bool wrapped = (my_flags & kInsWrapped) != 0;
     const bool failed = (my_flags & kInsFailed) != 0;
@@ -324,7 +336,7 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
       int carry = 0;
       if constexpr (WPR > 1) {
         int occ = 0;
-        for (int s = s_begin + lane; s < s_begin + kPerWarp; s += 32) occ += keys[s] != kEmptyKey;
+        for (int s = s_begin + lane; s < s_begin + kPerWarp; s += 32) occ += PairSlot<T>::key(pairs[s]) != kEmptyKey;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) occ += __shfl_xor_sync(kFull, occ, o);
         if (lane == 0) s_warp[warp] = occ;
@@ -336,7 +348,8 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
       bool count_err = false;
       for (int c0 = s_begin; c0 < s_begin + kPerWarp; c0 += 32) {
         const int s = c0 + lane;
-        const int key = keys[s];
+        const PW pr = pairs[s];
+        const int key = PairSlot<T>::key(pr);
         const bool occ = key != kEmptyKey;
         const unsigned m = __ballot_sync(kFull, occ);
         if (occ) {
@@ -344,7 +357,7 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
           const int64_t pos = static_cast<int64_t>(carry) + __popc(m & ((1u << lane) - 1u));
           if (pos < cnt) {
             p.c_colidx[base + pos] = key;
-            p.c_vals[base + pos] = vals[s];
+            p.c_vals[base + pos] = PairSlot<T>::val(pr);
           } else {
             count_err = true;
           }
@@ -364,7 +377,7 @@ __global__ void __launch_bounds__(32 * WPR * RPC, 1024 / (32 * WPR * RPC)) hash_
 template <typename T, int LOGT, int WPR, int RPC>
 void launch_bin(const RowPlan<T>& p, bool numeric, int bin, int num_sms, cudaStream_t s) {
   constexpr int kS = (1 << LOGT) + tail_slots(WPR);
-  const size_t smem = static_cast<size_t>(RPC) * kS * (sizeof(int) + (numeric ? sizeof(T) : 0));
+  const size_t smem = static_cast<size_t>(RPC) * kS * (numeric ? sizeof(typename PairSlot<T>::W) : sizeof(int));
   const int threads = 32 * WPR * RPC;
   auto kern = numeric ? hash_rows_kernel<T, LOGT, WPR, RPC, true> : hash_rows_kernel<T, LOGT, WPR, RPC, false>;
   static bool configured[2] = {false, false};
