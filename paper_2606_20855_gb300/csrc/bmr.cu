@@ -32,6 +32,7 @@
 // those rows); the rows it does not take are queued for the analysis kernel.
 // Its numeric pass is bmr_numeric_kernel, as for the binned rows.
 #include <climits>
+#include <type_traits>
 
 #include "ws_internal.cuh"
 
@@ -281,14 +282,54 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_symbolic_kernel(const
 // Staging slots of one warp: a row has at most kBmrMaxA * G products (the
 // lane groups of G lanes take kBmrMaxA stored A entries), so at most that
 // many entries; smaller groups need less shared memory and fit more warps.
+// Bulk asynchronous copy of a staged output segment from shared memory to C
+// (the copy engine of cp.async.bulk; addresses 16-byte aligned, size a
+// multiple of 16).  The issuing thread tracks its copies in bulk groups.
+__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst),
+               "r"(static_cast<uint32_t>(__cvta_generic_to_shared(ssrc))), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until every committed copy of this thread has read its source.
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// Waits until every committed copy of this thread is complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Orders this thread's earlier shared-memory writes before later bulk copies.
+__device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Writes the staged row (entries 0..cnt-1 at stage[pad + s]) to out[0..cnt-1]:
+// the 16-byte aligned middle by one bulk copy issued by lane 0, the up to
+// 16 / sizeof(V) - 1 entries on either side by single lanes.  `pad` is the
+// element offset of out within its 16-byte block, so stage[pad + s] and
+// out[s] share their alignment.
+// Rows shorter than kBulkMinEntries are copied by the lanes alone: there the
+// copy engine's latency, paid before the staging is reused, costs more than
+// the stores it saves.
+constexpr int kBulkMinEntries = 128;
+template <typename V>
+__device__ __forceinline__ void store_row(V* out, const V* stage, int pad, int cnt, int lane) {
+  constexpr int kPer = 16 / static_cast<int>(sizeof(V));
+  const int a = (kPer - pad) & (kPer - 1);        // first entry on a 16-byte boundary of out
+  const int b = ((pad + cnt) & ~(kPer - 1)) - pad;  // end of the last whole 16-byte block
+  if (cnt >= kBulkMinEntries && b > a) {
+    if (lane == 0) bulk_store(out + a, stage + pad + a, static_cast<uint32_t>((b - a) * sizeof(V)));
+    if (lane < a) out[lane] = stage[pad + lane];
+    const int t = lane - kPer;
+    if (t >= 0 && b + t < cnt) out[b + t] = stage[pad + b + t];
+  } else {
+    for (int s2 = lane; s2 < cnt; s2 += 32) out[s2] = stage[pad + s2];
+  }
+}
+
 template <int G>
 constexpr int numeric_cap() { return kBmrMaxA * G; }
 
 template <typename T, int G>
 constexpr size_t numeric_warp_bytes() {
-  return static_cast<size_t>(numeric_cap<G>()) * (4 + sizeof(T)) +
+  return (static_cast<size_t>(numeric_cap<G>()) + 4) * 4 + (static_cast<size_t>(numeric_cap<G>()) + 16 / sizeof(T)) * sizeof(T) +
          static_cast<size_t>(kHdrRows) * kBmrMaxA * (sizeof(long long) + sizeof(int) + sizeof(T)) +
-         static_cast<size_t>(kHdrRows) * (2 * sizeof(long long) + sizeof(int));
+         static_cast<size_t>(kHdrRows) * (2 * sizeof(long long) + 2 * sizeof(int));
 }
 
 template <typename T, int G>
@@ -304,18 +345,25 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
   constexpr int kCap = numeric_cap<G>();
   static_assert(kCap <= kBmrCap, "ranks fit the plan's 15 bits");
   unsigned char* ws = smem_raw + static_cast<size_t>(sub) * numeric_warp_bytes<T, G>();
+  // Staging of the sorted row, each array one 16-byte block longer so that
+  // entry s sits at pad + s with the alignment of C's entry.
+  constexpr int kValPer = 16 / static_cast<int>(sizeof(T));
+  static_assert(numeric_warp_bytes<T, G>() % 16 == 0, "every warp's staging starts on a 16-byte boundary");
   int* st_key = reinterpret_cast<int*>(ws);
-  T* st_val = reinterpret_cast<T*>(ws + static_cast<size_t>(kCap) * 4);
-  long long* h_b0 = reinterpret_cast<long long*>(ws + static_cast<size_t>(kCap) * (4 + sizeof(T)));
+  T* st_val = reinterpret_cast<T*>(ws + (static_cast<size_t>(kCap) + 4) * 4);
+  long long* h_b0 = reinterpret_cast<long long*>(ws + (static_cast<size_t>(kCap) + 4) * 4 +
+                                                 (static_cast<size_t>(kCap) + kValPer) * sizeof(T));
   T* h_a = reinterpret_cast<T*>(h_b0 + kEnt);
   int* h_len = reinterpret_cast<int*>(h_a + kEnt);
   long long* h_cbase = reinterpret_cast<long long*>(h_len + kEnt);  // C offset and nnz of each batch row
   long long* h_cnt = h_cbase + kHdrRows;
   int* h_row = reinterpret_cast<int*>(h_cnt + kHdrRows);
+  int* h_full = h_row + kHdrRows;  // 1: the row has kBmrMaxA stored entries whose B rows hold G entries each
 
   // hb (1..kHdrRows) rows per batch: fewer when the segment is too short to
   // give every warp of the grid a full batch.
   const int64_t warps = static_cast<int64_t>(gridDim.x) * kRowsPerCta;
+  bool bulk_pending = false;  // lane 0 has a bulk copy of the staging in flight
   for (int64_t r0 = (static_cast<int64_t>(blockIdx.x) * kRowsPerCta + sub) * hb; r0 < p.seg_len; r0 += warps * hb) {
     // Batch header: lane i < hb fetches row r0 + i.
     int na_l = 0;
@@ -348,6 +396,10 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
         h_a[e] = p.A.vals[ra + j];
       }
       h_len[e] = len;
+      // rows 2q (lanes 0..15) and 2q + 1 (lanes 16..31) of the batch
+      static_assert(kBmrMaxA == 16, "a batch row is a half warp here");
+      const unsigned fm = __ballot_sync(kFull, na == kBmrMaxA && len == G);
+      if (j == 0) h_full[i] = ((fm >> (lane & 16)) & 0xffffu) == 0xffffu;
     }
     __syncwarp();
     for (int i = 0; i < kHdrRows; ++i) {
@@ -357,64 +409,90 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, sizeof(T) == 8 ? 5 : 7) bmr_
       const long long want = h_cnt[i];
       const int cnt = static_cast<int>(want < kCap ? want : kCap);  // staging bounds every access
       if (lane == 0 && want > kCap) atomicOr(&p.sum->status, kErrCount);
+      int* out_key = p.c_colidx + cbase;
+      T* out_val = p.c_vals + cbase;
+      const int pk = static_cast<int>((reinterpret_cast<uintptr_t>(out_key) >> 2) & 3);
+      const int pv = static_cast<int>((reinterpret_cast<uintptr_t>(out_val) / sizeof(T)) & (kValPer - 1));
       const uint32_t* ranks2 = reinterpret_cast<const uint32_t*>(p.ranks + static_cast<int64_t>(row) * kBmrSlots);
-      int col[kSteps];
-      uint32_t rk2[kSteps / 2];  // ranks of steps q (low half) and q + kSteps / 2 (high half)
-      T val[kSteps];
-      uint32_t has_lo = 0;  // bit q: step q has a product
-#pragma unroll
-      for (int st = 0; st < kSteps; ++st) {
-        const int e = i * kBmrMaxA + st * kGroups + grp;
-        const bool has = gl < h_len[e];
-        col[st] = -1;
-        val[st] = T(0);
-        if (has) {
-          const long long b0 = h_b0[e];
-          col[st] = p.B.colidx[b0 + gl];
-          val[st] = p.B.vals[b0 + gl];  // scaled by the A value at the scatter
-        }
-        if (st < kSteps / 2) {
-          has_lo |= static_cast<uint32_t>(has) << st;
-        } else {
-          const int q = st - kSteps / 2;
-          rk2[q] = (((has_lo >> q) & 1u) || has) ? ranks2[rank_word<kSteps>(q, lane)] : 0u;
-        }
-      }
-      bool bad = false, repeats = false;
-#pragma unroll
-      for (int st = 0; st < kSteps; ++st) {
-        if (col[st] >= 0) {
-          const int rk = static_cast<int>(st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16);
-          const int r = rk & 0x7fff;
-          val[st] *= h_a[i * kBmrMaxA + st * kGroups + grp];
-          if (r >= cnt) {
-            bad = true;
-          } else if (rk & 0x8000) {
-            repeats = true;
-          } else {
-            st_key[r] = col[st];
-            st_val[r] = val[st];
-          }
-        }
-      }
-      if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
-      __syncwarp();
-      if (__any_sync(kFull, repeats)) {
+      // The row's products, their ranks, and the scatter into the staging.
+      // A full row (every step of every lane has a product) takes the same
+      // steps without the per-product tests.
+      auto scatter = [&](auto full_tag) {
+        constexpr bool kFullRow = decltype(full_tag)::value;
+        int col[kSteps];
+        uint32_t rk2[kSteps / 2];  // ranks of steps q (low half) and q + kSteps / 2 (high half)
+        T val[kSteps];
+        uint32_t has_lo = 0;  // bit q: step q has a product
 #pragma unroll
         for (int st = 0; st < kSteps; ++st) {
-          const int rk = static_cast<int>(st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16);
-          const int r = rk & 0x7fff;
-          if (col[st] >= 0 && (rk & 0x8000) && r < cnt) atomicAdd(&st_val[r], val[st]);
+          const int e = i * kBmrMaxA + st * kGroups + grp;
+          const bool has = kFullRow || gl < h_len[e];
+          col[st] = -1;
+          val[st] = T(0);
+          if (has) {
+            const long long b = h_b0[e] + gl;
+            col[st] = p.B.colidx[b];
+            val[st] = p.B.vals[b];  // scaled by the A value at the scatter
+          }
+          if (st < kSteps / 2) {
+            has_lo |= static_cast<uint32_t>(has) << st;
+          } else {
+            const int q = st - kSteps / 2;
+            rk2[q] = (kFullRow || ((has_lo >> q) & 1u) || has) ? ranks2[rank_word<kSteps>(q, lane)] : 0u;
+          }
         }
+        // The previous row's bulk copies must have read the staging.
+        if (lane == 0 && bulk_pending) bulk_wait_read();
         __syncwarp();
+        // Common case: rank below cnt with the repeat bit clear; the rest
+        // (repeated columns, and ranks out of range) after the first stores.
+        uint32_t rest = 0;
+#pragma unroll
+        for (int st = 0; st < kSteps; ++st) {
+          const uint32_t rk = st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16;
+          val[st] *= h_a[i * kBmrMaxA + st * kGroups + grp];
+          if (kFullRow || col[st] >= 0) {
+            if (rk < static_cast<uint32_t>(cnt)) {
+              st_key[pk + rk] = col[st];
+              st_val[pv + rk] = val[st];
+            } else {
+              rest |= 1u << st;
+            }
+          }
+        }
+        if (__any_sync(kFull, rest != 0)) {
+          __syncwarp();
+          bool bad = false;
+#pragma unroll
+          for (int st = 0; st < kSteps; ++st) {
+            if ((rest >> st) & 1u) {
+              const uint32_t rk = st < kSteps / 2 ? rk2[st] & 0xffffu : rk2[st - kSteps / 2] >> 16;
+              const uint32_t r = rk & 0x7fffu;
+              if ((rk & 0x8000u) && r < static_cast<uint32_t>(cnt)) {
+                atomicAdd(&st_val[pv + r], val[st]);
+              } else {
+                bad = true;
+              }
+            }
+          }
+          if (__any_sync(kFull, bad) && lane == 0) atomicOr(&p.sum->status, kErrCount);
+        }
+      };
+      if (h_full[i]) {
+        scatter(std::true_type{});
+      } else {
+        scatter(std::false_type{});
       }
-      for (int s2 = lane; s2 < cnt; s2 += 32) {
-        p.c_colidx[cbase + s2] = st_key[s2];
-        p.c_vals[cbase + s2] = st_val[s2];
-      }
+      fence_async_shared();
       __syncwarp();
+      store_row(out_key, st_key, pk, cnt, lane);
+      store_row(out_val, st_val, pv, cnt, lane);
+      bulk_pending = cnt >= kBulkMinEntries;
+      if (lane == 0 && bulk_pending) bulk_commit();
     }
+    __syncwarp();  // the next batch rewrites the headers
   }
+  if (lane == 0) bulk_wait_all();
 }
 
 // Grouped register bitmap rows: bin 0 (column range of at most kGrpWords * 32
@@ -777,7 +855,7 @@ __device__ __forceinline__ uint32_t plan_pre(uint32_t w) {
 
 template <typename T, int LOGW, int G>
 __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
-                                                                    int64_t ncols, int32_t* pending) {
+                                                                    int64_t ncols, int32_t* pending, int hb) {
   using S = PlanShape<LOGW>;
   constexpr int kGroups = 32 / G;
   constexpr int kSteps = kBmrMaxA / kGroups;  // steps of the one-warp numeric layout
@@ -799,8 +877,9 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
   int taken = 0;
   unsigned long long prod = 0;
 
-  for (int64_t r0 = static_cast<int64_t>(blockIdx.x) * kPlanHdrRows; r0 < ap.m;
-       r0 += static_cast<int64_t>(gridDim.x) * kPlanHdrRows) {
+  // hb (1..kPlanHdrRows) rows per batch: fewer when A has too few rows to
+  // give every CTA of one wave a full batch.
+  for (int64_t r0 = static_cast<int64_t>(blockIdx.x) * hb; r0 < ap.m; r0 += static_cast<int64_t>(gridDim.x) * hb) {
     __syncthreads();  // previous batch done with the header arrays (and the first bitmap clear)
     // Batch header: thread t reads stored A entry j = t % 16 of row r0 + t / 16
     // and the extent of its B row (rows with more than bmr_max_a entries are not read).
@@ -808,7 +887,7 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
       const int i = t / kBmrMaxA, j = t % kBmrMaxA;
       long long ra_l = 0;
       int na_l = 0;
-      if (lane < 2 && r0 + 2 * warp + lane < ap.m) {  // lanes 0, 1: the two rows of this warp
+      if (lane < 2 && 2 * warp + lane < hb && r0 + 2 * warp + lane < ap.m) {  // lanes 0, 1: the two rows of this warp
         const int64_t r = r0 + 2 * warp + lane;
         ra_l = p.A.rowptr[r];
         const long long n = p.A.rowptr[r + 1] - ra_l;
@@ -838,7 +917,7 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
       }
     }
     __syncthreads();
-    const int nrows = static_cast<int>(ap.m - r0 < kPlanHdrRows ? ap.m - r0 : kPlanHdrRows);
+    const int nrows = static_cast<int>(ap.m - r0 < hb ? ap.m - r0 : hb);
 #pragma unroll 1
     for (int i = 0; i < nrows; ++i) {
       const int64_t row = r0 + i;
@@ -847,90 +926,100 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
         if (t == 0) pending[atomicAdd(&p.sum->n_pending, 1)] = static_cast<int32_t>(row);
         continue;
       }
-      // Products of this thread: step st is numeric step s = 2 * st + warp.
-      int col[kMy];
-#pragma unroll
-      for (int st = 0; st < kMy; ++st) {
-        const unsigned long long h = h_ent[i * kBmrMaxA + (2 * st + warp) * kGroups + grp];
-        col[st] = gl < static_cast<int>(h >> kLenShift) ? p.B.colidx[(h & kPosMask) + gl] : -1;
-      }
-      if (i > 0) __syncthreads();  // the previous row's clear is complete
-      // Set the product bits; a product that finds its bit set repeats a column.
-      uint32_t dup = 0;
-#pragma unroll
-      for (int st = 0; st < kMy; ++st) {
-        if (col[st] >= 0) {
+      // A full row (kBmrMaxA stored entries, B rows of G entries each) takes
+      // the same steps without the per-product tests.
+      auto rank_row = [&](auto full_tag) {
+        constexpr bool kFullRow = decltype(full_tag)::value;
+        // Products of this thread: step st is numeric step s = 2 * st + warp.
+        int col[kMy];
+  #pragma unroll
+        for (int st = 0; st < kMy; ++st) {
+          const unsigned long long h = h_ent[i * kBmrMaxA + (2 * st + warp) * kGroups + grp];
+          col[st] = (kFullRow || gl < static_cast<int>(h >> kLenShift)) ? p.B.colidx[(h & kPosMask) + gl] : -1;
+        }
+        if (i > 0) __syncthreads();  // the previous row's clear is complete
+        // Set the product bits; a product that finds its bit set repeats a column.
+        uint32_t dup = 0;
+  #pragma unroll
+        for (int st = 0; st < kMy; ++st) {
+          if (kFullRow || col[st] >= 0) {
+            const uint32_t off = static_cast<uint32_t>(col[st]);
+            const uint32_t bit = 1u << (off & 31u);
+            if (atomicOr(bm + plan_bm<S>(off >> 5), bit) & bit) dup |= 1u << st;
+          }
+        }
+        __syncthreads();
+        // Sweep: local rank of the first column of each of this thread's words,
+        // two per register (word 2k low half, 2k + 1 high half).
+        uint32_t loc[(S::kWPT + 1) / 2];
+        uint32_t run = 0;
+        if constexpr (S::kWPT >= 4) {
+          const uint4* mine = reinterpret_cast<const uint4*>(bm) + t * (S::kWPT / 4);
+  #pragma unroll
+          for (int c = 0; c < S::kWPT / 4; ++c) {
+            const uint4 v = mine[S::kWPT == 32 ? (c ^ (t & 7)) : S::kWPT == 8 ? (c ^ ((t >> 2) & 1)) : c];
+            const uint32_t r1 = run + __popc(v.x);
+            const uint32_t r2 = r1 + __popc(v.y);
+            const uint32_t r3 = r2 + __popc(v.z);
+            loc[2 * c] = run | (r1 << 16);
+            loc[2 * c + 1] = r2 | (r3 << 16);
+            run = r3 + __popc(v.w);
+          }
+        } else {
+          const uint2 v = reinterpret_cast<const uint2*>(bm)[t];
+          loc[0] = __popc(v.x) << 16;
+          run = __popc(v.x) + __popc(v.y);
+        }
+        uint32_t incl = run;
+  #pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(kFull, incl, o);
+          if (lane >= o) incl += y;
+        }
+        if (lane == 31) s_cnt[warp] = static_cast<int>(incl);
+        // Word ranks within this warp's half (both halves of a register: no carry, every rank <= kBmrCap).
+        const uint32_t base = incl - run;
+        const uint32_t base2 = base | (base << 16);
+        if constexpr (S::kWPT == 32) {
+          uint4* pm = reinterpret_cast<uint4*>(pre) + t * 4;
+  #pragma unroll
+          for (int q = 0; q < 4; ++q)
+            pm[q ^ ((t >> 1) & 3)] = make_uint4(loc[4 * q] + base2, loc[4 * q + 1] + base2, loc[4 * q + 2] + base2,
+                                                loc[4 * q + 3] + base2);
+        } else if constexpr (S::kWPT == 8) {
+          reinterpret_cast<uint4*>(pre)[t] = make_uint4(loc[0] + base2, loc[1] + base2, loc[2] + base2, loc[3] + base2);
+        } else {
+          reinterpret_cast<uint32_t*>(pre)[t] = loc[0] + base2;
+        }
+        __syncthreads();
+        const uint32_t lower = static_cast<uint32_t>(s_cnt[0]);  // entries in warp 0's half of the columns
+        // Rank of this thread's step st product: its word's rank within its
+        // half, warp 0's count for a column of warp 1's half, and the bits below
+        // it in its word.
+        auto rank_of = [&](int st) -> uint32_t {
+          if (!kFullRow && col[st] < 0) return 0u;
           const uint32_t off = static_cast<uint32_t>(col[st]);
-          const uint32_t bit = 1u << (off & 31u);
-          if (atomicOr(bm + plan_bm<S>(off >> 5), bit) & bit) dup |= 1u << st;
+          const uint32_t w = off >> 5;
+          const uint32_t half = (w >> (LOGW - 1)) & 1u;
+          return (pre[plan_pre<S>(w)] + (half ? lower : 0u) +
+                  __popc(bm[plan_bm<S>(w)] & ((1u << (off & 31u)) - 1u))) |
+                 ((dup << (15 - st)) & 0x8000u);
+        };
+        uint32_t* ranks32 = reinterpret_cast<uint32_t*>(p.ranks + row * kBmrSlots);
+        if constexpr (kHalf % 2 == 0) {
+          // numeric steps s and s + kHalf (st and st + kHalf / 2 here) share a rank word
+  #pragma unroll
+          for (int st = 0; st < kHalf / 2; ++st)
+            ranks32[((2 * st + warp) << 5) | lane] = rank_of(st) | (rank_of(st + kHalf / 2) << 16);
+        } else {
+          // one step per warp (G = 4): warp w fills half w of rank word 0
+          p.ranks[row * kBmrSlots + 2 * lane + warp] = static_cast<uint16_t>(rank_of(0));
         }
-      }
-      __syncthreads();
-      // Sweep: local rank of the first column of each of this thread's words,
-      // two per register (word 2k low half, 2k + 1 high half).
-      uint32_t loc[(S::kWPT + 1) / 2];
-      uint32_t run = 0;
-      if constexpr (S::kWPT >= 4) {
-        const uint4* mine = reinterpret_cast<const uint4*>(bm) + t * (S::kWPT / 4);
-#pragma unroll
-        for (int c = 0; c < S::kWPT / 4; ++c) {
-          const uint4 v = mine[S::kWPT == 32 ? (c ^ (t & 7)) : S::kWPT == 8 ? (c ^ ((t >> 2) & 1)) : c];
-          const uint32_t r1 = run + __popc(v.x);
-          const uint32_t r2 = r1 + __popc(v.y);
-          const uint32_t r3 = r2 + __popc(v.z);
-          loc[2 * c] = run | (r1 << 16);
-          loc[2 * c + 1] = r2 | (r3 << 16);
-          run = r3 + __popc(v.w);
-        }
-      } else {
-        const uint2 v = reinterpret_cast<const uint2*>(bm)[t];
-        loc[0] = __popc(v.x) << 16;
-        run = __popc(v.x) + __popc(v.y);
-      }
-      uint32_t incl = run;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += y;
-      }
-      if (lane == 31) s_cnt[warp] = static_cast<int>(incl);
-      // Word ranks within this warp's half (both halves of a register: no carry, every rank <= kBmrCap).
-      const uint32_t base = incl - run;
-      const uint32_t base2 = base | (base << 16);
-      if constexpr (S::kWPT == 32) {
-        uint4* pm = reinterpret_cast<uint4*>(pre) + t * 4;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          pm[q ^ ((t >> 1) & 3)] = make_uint4(loc[4 * q] + base2, loc[4 * q + 1] + base2, loc[4 * q + 2] + base2,
-                                              loc[4 * q + 3] + base2);
-      } else if constexpr (S::kWPT == 8) {
-        reinterpret_cast<uint4*>(pre)[t] = make_uint4(loc[0] + base2, loc[1] + base2, loc[2] + base2, loc[3] + base2);
-      } else {
-        reinterpret_cast<uint32_t*>(pre)[t] = loc[0] + base2;
-      }
-      __syncthreads();
-      const uint32_t lower = static_cast<uint32_t>(s_cnt[0]);  // entries in warp 0's half of the columns
-      // Rank of this thread's step st product: its word's rank within its
-      // half, warp 0's count for a column of warp 1's half, and the bits below
-      // it in its word.
-      auto rank_of = [&](int st) -> uint32_t {
-        if (col[st] < 0) return 0u;
-        const uint32_t off = static_cast<uint32_t>(col[st]);
-        const uint32_t w = off >> 5;
-        const uint32_t half = (w >> (LOGW - 1)) & 1u;
-        return (pre[plan_pre<S>(w)] + (half ? lower : 0u) +
-                __popc(bm[plan_bm<S>(w)] & ((1u << (off & 31u)) - 1u))) |
-               ((dup << (15 - st)) & 0x8000u);
       };
-      uint32_t* ranks32 = reinterpret_cast<uint32_t*>(p.ranks + row * kBmrSlots);
-      if constexpr (kHalf % 2 == 0) {
-        // numeric steps s and s + kHalf (st and st + kHalf / 2 here) share a rank word
-#pragma unroll
-        for (int st = 0; st < kHalf / 2; ++st)
-          ranks32[((2 * st + warp) << 5) | lane] = rank_of(st) | (rank_of(st + kHalf / 2) << 16);
+      if (hr.x == kBmrMaxA && hr.y == kBmrMaxA * G) {
+        rank_row(std::true_type{});
       } else {
-        // one step per warp (G = 4): warp w fills half w of rank word 0
-        p.ranks[row * kBmrSlots + 2 * lane + warp] = static_cast<uint16_t>(rank_of(0));
+        rank_row(std::false_type{});
       }
       __syncthreads();
       // Clear this thread's words (conflict-free, the sweep's order).
@@ -1014,9 +1103,12 @@ void launch_plan_g(const RowPlan<T>& p, const AnalyzeParams& ap, int64_t ncols, 
   const size_t smem = PlanShape<LOGW>::kBytes;
   static int per_sm = 0;
   if (per_sm == 0) per_sm = occupancy(bmr_plan_kernel<T, LOGW, G>, kPlanThreads, smem);
-  constexpr int64_t kPerCta = kPlanHdrRows;
-  const int64_t grid = clamp_grid((ap.m + kPerCta - 1) / kPerCta, num_sms, per_sm);
-  bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), kPlanThreads, smem, s>>>(p, ap, ncols, pending);
+  const int64_t wave = static_cast<int64_t>(num_sms) * per_sm;
+  int64_t hb = (ap.m + wave - 1) / wave;
+  hb = hb < 1 ? 1 : (hb > kPlanHdrRows ? kPlanHdrRows : hb);
+  const int64_t grid = clamp_grid((ap.m + hb - 1) / hb, num_sms, per_sm);
+  bmr_plan_kernel<T, LOGW, G><<<static_cast<int>(grid), kPlanThreads, smem, s>>>(p, ap, ncols, pending,
+                                                                                 static_cast<int>(hb));
 }
 
 template <typename T, int G>
