@@ -313,13 +313,16 @@ ws_status_t ws_spgemm_plan_info(ws_csr_t C, int64_t* info, int n);
  *   key 7: widest column range of a heavy row that uses the wide-bitmap path
  *          (default and maximum 1048576; 0 disables it)
  *   key 8: elementwise operations, lanes per row chunk: -1 (default:
- *          automatic, 1 for rows averaging under 64 merged entries, 64
- *          otherwise), 1 (one thread merges a chunk entry by entry), 4, 8,
- *          16 or 32 (a lane group merges windows of that many entries), 0
- *          (lane group sized from the mean row length), 64 (a warp per
- *          64-entry chunk ranks every entry by binary search)
+ *          automatic, 2 for rows averaging under 64 merged entries, 64
+ *          otherwise), 1 (one thread merges a chunk entry by entry from
+ *          global memory), 2 (the same from shared-memory copies of the
+ *          input runs of a warp's 32 chunks, chunks of at most 16 merged
+ *          entries), 4, 8, 16 or 32 (a lane group merges windows of that
+ *          many entries), 0 (lane group sized from the mean row length), 64
+ *          (a warp per 64-entry chunk ranks every entry by binary search)
  *   key 9: elementwise operations with one lane per chunk: merged entries
- *          per chunk (default 64, range [2, 1048576])
+ *          per chunk (default 64, range [2, 1048576]; with key 8 = 2 at
+ *          most 16 are used)
  * Returns WS_ERR_INVALID_ARG for an unknown key or out-of-range value.
  */
 ws_status_t ws_set_tuning(int key, int64_t value);

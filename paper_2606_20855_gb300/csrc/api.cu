@@ -153,6 +153,7 @@ struct Plan {
   int32_t* ew_chunk_row = nullptr;
   int64_t* ew_chunk_off = nullptr;
   int64_t* ew_chunk_split = nullptr;
+  int64_t* ew_chunk_bpos = nullptr;
   int64_t* ew_partials = nullptr;
   int32_t* rcd_scnt = nullptr;
   int32_t* rcd_mega = nullptr;
@@ -557,7 +558,8 @@ ws_status_t carve_ewise(Plan* pl, int64_t m, int64_t nc_max, cudaStream_t s) {
   const size_t o_begin = off; off = align_up(off + 8 * static_cast<size_t>(m + 1), 256);
   const size_t o_row = off; off = align_up(off + 4 * static_cast<size_t>(nc_max), 256);
   const size_t o_off = off; off = align_up(off + 8 * static_cast<size_t>(nc_max + 1), 256);
-  const size_t o_split = off; off = align_up(off + 8 * static_cast<size_t>(nc_max), 256);
+  const size_t o_split = off; off = align_up(off + 8 * static_cast<size_t>(nc_max + 1), 256);
+  const size_t o_bpos = off; off = align_up(off + 8 * static_cast<size_t>(nc_max + 1), 256);
   const size_t o_part = off; off = align_up(off + 8 * static_cast<size_t>(nb + 1), 256);
   ws_status_t st = pl->ew.reserve(off, s);
   if (st != WS_OK) return st;
@@ -567,6 +569,7 @@ ws_status_t carve_ewise(Plan* pl, int64_t m, int64_t nc_max, cudaStream_t s) {
   pl->ew_chunk_row = reinterpret_cast<int32_t*>(b + o_row);
   pl->ew_chunk_off = reinterpret_cast<int64_t*>(b + o_off);
   pl->ew_chunk_split = reinterpret_cast<int64_t*>(b + o_split);
+  pl->ew_chunk_bpos = reinterpret_cast<int64_t*>(b + o_bpos);
   pl->ew_partials = reinterpret_cast<int64_t*>(b + o_part);
   return WS_OK;
 }
@@ -584,6 +587,7 @@ EwisePlan<T> make_ewise(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* C, const
   p.chunk_row = pl->ew_chunk_row;
   p.chunk_off = pl->ew_chunk_off;
   p.chunk_split = pl->ew_chunk_split;
+  p.chunk_bpos = pl->ew_chunk_bpos;
   p.nc_max = pl->ew_nc_max;
   p.partials = pl->ew_partials;
   p.sum = pl->dsum;
@@ -603,12 +607,14 @@ ws_status_t ewise_symbolic_impl(const ws_csr_s* A, const ws_csr_s* B, ws_csr_s* 
   pl->num_launches = 0;
   pl->ew_op = op;
   const int64_t merged = A->nnz + B->nnz;
-  // automatic: one thread per chunk for short rows (power-law graphs), a warp
-  // per 64-position chunk once rows average a whole chunk
+  // automatic: a lane per chunk of a warp-staged tile for short rows
+  // (power-law graphs), a warp per 64-position chunk once rows average a
+  // whole chunk
   const bool long_rows = m > 0 && merged >= static_cast<int64_t>(kEwiseRankChunk) * m;
   pl->ew_group = g_ewise_lanes > 0 ? g_ewise_lanes
-               : g_ewise_lanes == 0 ? ewise_group_for(m, merged) : (long_rows ? kEwiseRankGroup : 1);
+               : g_ewise_lanes == 0 ? ewise_group_for(m, merged) : (long_rows ? kEwiseRankGroup : kEwiseTileGroup);
   pl->ew_diag = pl->ew_group == 1 ? g_ewise_diag
+              : pl->ew_group == kEwiseTileGroup ? (g_ewise_diag < kEwiseTileDiag ? g_ewise_diag : kEwiseTileDiag)
               : pl->ew_group == kEwiseRankGroup ? kEwiseRankChunk : 16 * static_cast<int64_t>(pl->ew_group);
   pl->ew_nc_max = m + merged / pl->ew_diag + 1;  // row i has at most 1 + len_i / diag chunks
   ws_status_t st = carve_ewise(pl, m, pl->ew_nc_max, s);
@@ -1400,9 +1406,9 @@ ws_status_t ws_set_tuning(int key, int64_t value) {
       g_wb_span = value;
       return WS_OK;
     case 8:
-      if (value != -1 && value != 0 && value != 1 && value != 4 && value != 8 && value != 16 && value != 32 &&
-          value != kEwiseRankGroup)
-        return fail(WS_ERR_INVALID_ARG, "elementwise lanes per chunk must be -1, 0, 1, 4, 8, 16, 32 or 64");
+      if (value != -1 && value != 0 && value != 1 && value != kEwiseTileGroup && value != 4 && value != 8 &&
+          value != 16 && value != 32 && value != kEwiseRankGroup)
+        return fail(WS_ERR_INVALID_ARG, "elementwise lanes per chunk must be -1, 0, 1, 2, 4, 8, 16, 32 or 64");
       g_ewise_lanes = static_cast<int>(value);
       return WS_OK;
     case 9:

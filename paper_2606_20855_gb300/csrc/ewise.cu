@@ -330,7 +330,7 @@ __device__ int64_t merge_add_fill(const int32_t* a, const T* va, int64_t na, con
 template <bool FILL, typename T>
 __device__ __forceinline__ void chunk_bounds(const EwisePlan<T>& p, int64_t c, const int32_t* a, int64_t na,
                                              const int32_t* b, int64_t nb, int64_t d0, int64_t d1, int64_t* i0,
-                                             int64_t* j0, int64_t* i1, int64_t* j1) {
+                                             int64_t* j0, int64_t* i1, int64_t* j1, bool writer) {
   auto decode = [&](int64_t d, int64_t code, int64_t* i, int64_t* j) {
     const int64_t lo = d - nb > 0 ? d - nb : 0, hi = d < na ? d : na;
     const int64_t x = code >> 1;
@@ -341,7 +341,7 @@ __device__ __forceinline__ void chunk_bounds(const EwisePlan<T>& p, int64_t c, c
   if constexpr (!FILL) {
     if (d0 > 0) merge_split(a, na, b, nb, d0, i0, j0);
     if (d1 < na + nb) merge_split(a, na, b, nb, d1, i1, j1);
-    if (threadIdx.x % p.group == 0) p.chunk_split[c] = 2 * *i0 + (*j0 - (d0 - *i0));
+    if (writer) p.chunk_split[c] = 2 * *i0 + (*j0 - (d0 - *i0));
   } else {
     decode(d0, p.chunk_split[c], i0, j0);
     if (d1 < na + nb) decode(d1, p.chunk_split[c + 1], i1, j1);  // the next chunk belongs to this row
@@ -370,7 +370,7 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(
     const int64_t d0 = k * p.diag;
     const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
     int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
-    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1);
+    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1, threadIdx.x % p.group == 0);
     if constexpr (FILL) {
       const int64_t o0 = p.chunk_off[c];
       const int64_t cap = p.chunk_off[c + 1] - o0;
@@ -387,6 +387,135 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_seq_kernel(
     } else {
       p.chunk_off[c + 1] = merge_seq<T, OP, false>(a + i0, nullptr, i1 - i0, b + j0, nullptr, j1 - j0, nullptr, &bad);
     }
+  }
+  if (bad) atomicOr(&p.sum->status, kErrCount);
+}
+
+// Warp-staged tiles: a warp takes 32 consecutive chunks, one per lane.  The
+// chunks' parts of A and of B are contiguous runs of A's and B's arrays
+// (consecutive chunks of a row continue each other; the rows between two
+// chunks are empty), so the warp first copies the two runs into shared
+// memory with coalesced loads; every lane then merges its chunk from there,
+// with no dependent global loads in the merge loop.  A lane whose bounds
+// fall outside the staged runs (only if the inputs changed since the
+// symbolic pass) merges from global memory; the count check then reports it.
+constexpr int kTileWarps = 4;
+constexpr int kTileCap = 32 * kEwiseTileDiag;  // staged entries per list and warp
+
+// Values are staged for the union's fill only: an intersection reads the
+// values of its (few) equal pairs from global memory.
+template <int OP, bool FILL>
+constexpr bool tile_stages_values() { return FILL && OP == kEwiseAdd; }
+template <typename T, int OP, bool FILL>
+constexpr size_t tile_warp_bytes() {
+  return 2 * static_cast<size_t>(kTileCap) * (sizeof(int32_t) + (tile_stages_values<OP, FILL>() ? sizeof(T) : 0));
+}
+
+template <typename T, int OP, bool FILL>
+__global__ void __launch_bounds__(32 * kTileWarps) ew_tile_kernel(const EwisePlan<T> p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr bool kVals = tile_stages_values<OP, FILL>();
+  // per warp: A values, B values (when staged), then A columns, B columns
+  unsigned char* ws = smem_raw + static_cast<size_t>(warp) * tile_warp_bytes<T, OP, FILL>();
+  T* sva = reinterpret_cast<T*>(ws);
+  T* svb = sva + (kVals ? kTileCap : 0);
+  int32_t* sca = reinterpret_cast<int32_t*>(svb + (kVals ? kTileCap : 0));
+  int32_t* scb = sca + kTileCap;
+  const int64_t nc = p.chunk_begin[p.m];
+  bool bad = false;
+  const bool vec = ((reinterpret_cast<uintptr_t>(p.c_colidx) | reinterpret_cast<uintptr_t>(p.c_vals)) & 15u) == 0;
+  const int64_t ntiles = (p.nc_max + 31) / 32;
+  for (int64_t tile = static_cast<int64_t>(blockIdx.x) * kTileWarps + warp; tile < ntiles;
+       tile += static_cast<int64_t>(gridDim.x) * kTileWarps) {
+    const int64_t c = tile * 32 + lane;
+    if (!FILL && c >= nc && c < p.nc_max) p.chunk_off[c + 1] = 0;
+    if (!FILL && c == nc) {  // end positions, read as the bounds after the last chunk
+      p.chunk_split[nc] = p.A.rowptr[p.m];
+      p.chunk_bpos[nc] = p.B.rowptr[p.m];
+    }
+    const bool valid = c < nc;
+    const unsigned vmask = __ballot_sync(kFull, valid);
+    if (vmask == 0u) continue;  // past the last chunk (the counts above are zeroed all the same)
+    // The chunk's parts of A and B as absolute positions [ga0, ga1), [gb0, gb1).
+    int64_t ga0 = 0, ga1 = 0, gb0 = 0, gb1 = 0;
+    if (valid) {
+      if constexpr (FILL) {
+        // kept by the symbolic pass; chunk c + 1 (or the end) bounds chunk c
+        ga0 = p.chunk_split[c];
+        gb0 = p.chunk_bpos[c];
+        ga1 = p.chunk_split[c + 1];
+        gb1 = p.chunk_bpos[c + 1];
+        // A changed input could leave the bounds out of order or outside the
+        // lists: clamp them (the count check then reports the difference).
+        const int64_t a_end = p.A.rowptr[p.m], b_end = p.B.rowptr[p.m];
+        ga0 = ga0 < 0 ? 0 : (ga0 > a_end ? a_end : ga0);
+        ga1 = ga1 < ga0 ? ga0 : (ga1 > a_end ? a_end : ga1);
+        gb0 = gb0 < 0 ? 0 : (gb0 > b_end ? b_end : gb0);
+        gb1 = gb1 < gb0 ? gb0 : (gb1 > b_end ? b_end : gb1);
+      } else {
+        const int32_t row = p.chunk_row[c];
+        const int64_t k = c - p.chunk_begin[row];
+        const int64_t a0 = p.A.rowptr[row], na = p.A.rowptr[row + 1] - a0;
+        const int64_t b0 = p.B.rowptr[row], nb = p.B.rowptr[row + 1] - b0;
+        const int64_t d0 = k * p.diag;
+        const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
+        int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
+        chunk_bounds<false>(p, c, p.A.colidx + a0, na, p.B.colidx + b0, nb, d0, d1, &i0, &j0, &i1, &j1, false);
+        ga0 = a0 + i0;
+        ga1 = a0 + i1;
+        gb0 = b0 + j0;
+        gb1 = b0 + j1;
+        p.chunk_split[c] = ga0;
+        p.chunk_bpos[c] = gb0;
+      }
+    }
+    // The tile's runs: from the first lane's start to the last valid lane's end.
+    const int last = 31 - __clz(vmask);
+    const int64_t alo = __shfl_sync(kFull, ga0, 0), ahi = __shfl_sync(kFull, ga1, last);
+    const int64_t blo = __shfl_sync(kFull, gb0, 0), bhi = __shfl_sync(kFull, gb1, last);
+    const bool staged = ahi - alo <= kTileCap && bhi - blo <= kTileCap && ahi >= alo && bhi >= blo;
+    if (staged) {
+      const int n_a = static_cast<int>(ahi - alo), n_b = static_cast<int>(bhi - blo);
+      for (int t = lane; t < n_a; t += 32) {
+        sca[t] = p.A.colidx[alo + t];
+        if constexpr (kVals) sva[t] = p.A.vals[alo + t];
+      }
+      for (int t = lane; t < n_b; t += 32) {
+        scb[t] = p.B.colidx[blo + t];
+        if constexpr (kVals) svb[t] = p.B.vals[blo + t];
+      }
+    }
+    __syncwarp();
+    if (valid) {
+      const bool mine = staged && ga0 >= alo && ga1 <= ahi && gb0 >= blo && gb1 <= bhi;
+      const int64_t na = ga1 - ga0, nb = gb1 - gb0;
+      // The same merge for staged lists and (after a changed input) for the
+      // global arrays; separate calls keep the staged one on shared-memory loads.
+      auto merge = [&](const int32_t* a, const T* va, const int32_t* b, const T* vb) {
+        if constexpr (FILL) {
+          const int64_t o0 = p.chunk_off[c];
+          const int64_t cap = p.chunk_off[c + 1] - o0;
+          int64_t n;
+          if constexpr (OP == kEwiseAdd) {
+            n = merge_add_fill<T>(a, va, na, b, vb, nb, p.c_colidx + o0, p.c_vals + o0, cap, o0, vec, &bad);
+          } else {
+            SeqWriter<T> w(p.c_colidx + o0, p.c_vals + o0, cap, o0, vec);
+            n = merge_seq<T, OP, true>(a, va, na, b, vb, nb, &w, &bad);
+          }
+          if (n != cap) bad = true;
+        } else {
+          p.chunk_off[c + 1] = merge_seq<T, OP, false>(a, nullptr, na, b, nullptr, nb, nullptr, &bad);
+        }
+      };
+      if (mine) {
+        merge(sca + (ga0 - alo), kVals ? sva + (ga0 - alo) : p.A.vals + ga0, scb + (gb0 - blo),
+              kVals ? svb + (gb0 - blo) : p.B.vals + gb0);
+      } else {
+        merge(p.A.colidx + ga0, p.A.vals + ga0, p.B.colidx + gb0, p.B.vals + gb0);
+      }
+    }
+    __syncwarp();  // the next tile rewrites the staging
   }
   if (bad) atomicOr(&p.sum->status, kErrCount);
 }
@@ -437,7 +566,7 @@ __global__ void __launch_bounds__(kEwThreads, FILL ? 4 : 6) ew_merge_kernel(cons
     const int64_t d0 = k * p.diag;
     const int64_t d1 = d0 + p.diag < na + nb ? d0 + p.diag : na + nb;
     int64_t i0 = 0, j0 = 0, i1 = na, j1 = nb;
-    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1);
+    chunk_bounds<FILL>(p, c, a, na, b, nb, d0, d1, &i0, &j0, &i1, &j1, threadIdx.x % p.group == 0);
     if constexpr (FILL) {
       const int64_t o0 = p.chunk_off[c];
       const int64_t cap = p.chunk_off[c + 1] - o0;
@@ -681,6 +810,19 @@ void launch_merge_g(const EwisePlan<T>& p, int num_sms, cudaStream_t s) {
   }
   if (p.group == 1) {
     ew_merge_seq_kernel<T, OP, FILL><<<grid_for(p.nc_max, kEwThreads, num_sms, 8), kEwThreads, 0, s>>>(p);
+    return;
+  }
+  if (p.group == kEwiseTileGroup) {
+    constexpr size_t smem = kTileWarps * tile_warp_bytes<T, OP, FILL>();
+    static bool configured = false;
+    if (!configured) {
+      cudaFuncSetAttribute(ew_tile_kernel<T, OP, FILL>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      configured = true;
+    }
+    int per_sm = 0;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ew_tile_kernel<T, OP, FILL>, 32 * kTileWarps, smem);
+    const int grid = grid_for((p.nc_max + 31) / 32, kTileWarps, num_sms, per_sm > 0 ? per_sm : 1);
+    ew_tile_kernel<T, OP, FILL><<<grid, 32 * kTileWarps, smem, s>>>(p);
     return;
   }
   switch (p.group) {

@@ -168,6 +168,8 @@ struct RowPlan {
 constexpr int kEwiseAdd = 1;  // SpAdd: pattern union, values added
 constexpr int kEwiseMul = 2;  // Hadamard product: pattern intersection, values multiplied
 constexpr int kEwiseRankGroup = 64;  // EwisePlan::group of the warp-per-chunk ranking kernels
+constexpr int kEwiseTileGroup = 2;   // EwisePlan::group of the warp-staged tile kernels (a lane per chunk)
+constexpr int kEwiseTileDiag = 16;   // their largest chunk (merged positions)
 constexpr int kEwiseRankChunk = 64;  // their merged positions per chunk
 
 template <typename T>
@@ -181,12 +183,15 @@ struct EwisePlan {
   int64_t* chunk_begin;  // [m + 1]: first chunk of each row (chunks per row, then scanned in place)
   int32_t* chunk_row;    // [nc_max]: row of each chunk
   int64_t* chunk_off;    // [nc_max + 1]: C offset of each chunk (counts, then scanned in place)
-  int64_t* chunk_split;  // [nc_max]: 2 * (A entries before the chunk) + (1 if an equal pair straddles its start)
+  int64_t* chunk_split;  // [nc_max + 1]: 2 * (A entries before the chunk) + (1 if an equal pair straddles its start);
+                         // warp-staged tiles: the chunk's first position in A's arrays ([nc]: the end of A)
+  int64_t* chunk_bpos;   // [nc_max + 1]: warp-staged tiles: the chunk's first position in B's arrays
   int64_t nc_max;        // bound on the number of chunks: m + (nnz(A) + nnz(B)) / diag + 1
   int64_t* partials;     // scan scratch for max(m, nc_max) entries
   DevSummary* sum;
   int64_t diag;          // merged positions per chunk
-  int group;             // lanes per chunk (1: one thread merges entry by entry; 4, 8, 16, 32: windows;
+  int group;             // lanes per chunk (1: one thread merges entry by entry; kEwiseTileGroup: the same
+                         // from shared-memory copies of a warp's 32 chunks; 4, 8, 16, 32: windows;
                          // kEwiseRankGroup: a warp per chunk ranks every entry by binary search)
   int op;                // kEwiseAdd or kEwiseMul
 };

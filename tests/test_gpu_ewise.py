@@ -53,10 +53,11 @@ def check(A, B, op, validate=False):
     return info
 
 
-# lanes per chunk: 1 (one thread per chunk), 0 (lane groups of 4..32 sized
-# from the mean row length) and 64 (a warp per 64-position chunk ranking every
-# entry by binary search)
-LANES = [1, 0, 64]
+# lanes per chunk: 1 (one thread per chunk), 2 (one lane per chunk of a
+# warp-staged tile of 32 chunks), 0 (lane groups of 4..32 sized from the mean
+# row length) and 64 (a warp per 64-position chunk ranking every entry by
+# binary search)
+LANES = [1, 2, 0, 64]
 
 
 @pytest.mark.parametrize("lanes", LANES)
@@ -104,7 +105,8 @@ def _long_rows(m, n, lens, rng, overlap):
     return build(ra), build(rb)
 
 
-@pytest.mark.parametrize("lanes,chunk", [(1, 64), (1, 2), (1, 7), (0, 64), (32, 64), (64, 64), (-1, 64)])
+@pytest.mark.parametrize("lanes,chunk", [(1, 64), (1, 2), (1, 7), (2, 16), (2, 2), (2, 7), (0, 64), (32, 64),
+                                         (64, 64), (-1, 64)])
 @pytest.mark.parametrize("op", OPS)
 @pytest.mark.parametrize("overlap", [0.0, 0.5, 1.0])
 def test_long_rows_many_chunks(overlap, op, lanes, chunk):
