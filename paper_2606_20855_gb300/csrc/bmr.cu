@@ -803,7 +803,9 @@ __global__ void __launch_bounds__(32 * kRowsPerCta, 6) bmr_group_numeric_kernel(
 // stores the rank (within its warp's half of the columns) of the first
 // column of each of its words.  A product's rank is then that word rank,
 // plus warp 0's count for a column of warp 1's half, plus the bits below it
-// in its word; the sweep's chunk order clears the bitmap for the next row.
+// in its word.  The bitmap is cleared for the next row by a bulk copy of a
+// zero block (the copy engine, tracked by an mbarrier), so the shared-memory
+// pipe the rest of the row is bound by does no clearing stores.
 //
 // Row headers (the B row extent of every stored A entry) are fetched for
 // kPlanHdrRows rows at a time.
@@ -853,6 +855,31 @@ __device__ __forceinline__ uint32_t plan_pre(uint32_t w) {
   }
 }
 
+// Zero block the planning pass copies over its bitmap after each row.
+static __device__ __align__(128) uint4 g_plan_zero[2048 / 4];
+__device__ __forceinline__ uint32_t smem_u32(const void* ptr) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(ptr));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_copy(uint64_t* bar, void* dst, const void* src, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+// Waits (bounded) for the phase `parity` of the barrier; false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (int it = 0; it < (1 << 20); ++it) {
+    uint32_t done;
+    asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+                 : "=r"(done) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
 template <typename T, int LOGW, int G>
 __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPlan<T> p, const AnalyzeParams ap,
                                                                     int64_t ncols, int32_t* pending, int hb) {
@@ -870,9 +897,16 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
   unsigned long long* h_ent = reinterpret_cast<unsigned long long*>(smem_raw + static_cast<size_t>(S::kWords) * 6);
   int4* h_row = reinterpret_cast<int4*>(h_ent + kPlanThreads);
   __shared__ int s_cnt[2];
+  __shared__ __align__(8) uint64_t s_mbar;
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int grp = lane / G, gl = lane % G;
   for (int i = t; i < S::kWords / 4; i += kPlanThreads) reinterpret_cast<uint4*>(bm)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (t == 0) {
+    mbar_init(&s_mbar, 1);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  uint32_t mphase = 0;
+  bool clr_pending = false;
   const long long words = (ncols + 31) >> 5;
   int taken = 0;
   unsigned long long prod = 0;
@@ -937,7 +971,11 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
           const unsigned long long h = h_ent[i * kBmrMaxA + (2 * st + warp) * kGroups + grp];
           col[st] = (kFullRow || gl < static_cast<int>(h >> kLenShift)) ? p.B.colidx[(h & kPosMask) + gl] : -1;
         }
-        if (i > 0) __syncthreads();  // the previous row's clear is complete
+        if (clr_pending) {  // the previous row's clear is complete
+        if (!mbar_wait(&s_mbar, mphase) && t == 0) atomicOr(&p.sum->status, kErrCount);
+        mphase ^= 1u;
+        clr_pending = false;
+      }
         // Set the product bits; a product that finds its bit set repeats a column.
         uint32_t dup = 0;
   #pragma unroll
@@ -1021,16 +1059,10 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
       } else {
         rank_row(std::false_type{});
       }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the bitmap reads before the copy over it
       __syncthreads();
-      // Clear this thread's words (conflict-free, the sweep's order).
-      if constexpr (S::kWPT >= 4) {
-        uint4* mine = reinterpret_cast<uint4*>(bm) + t * (S::kWPT / 4);
-#pragma unroll
-        for (int c = 0; c < S::kWPT / 4; ++c)
-          mine[S::kWPT == 32 ? (c ^ (t & 7)) : S::kWPT == 8 ? (c ^ ((t >> 2) & 1)) : c] = make_uint4(0u, 0u, 0u, 0u);
-      } else {
-        reinterpret_cast<uint2*>(bm)[t] = make_uint2(0u, 0u);
-      }
+      if (t == 0) mbar_expect_copy(&s_mbar, bm, g_plan_zero, static_cast<uint32_t>(S::kWords * 4));
+      clr_pending = true;
       if (t == 0) {
         p.c_rowptr[row + 1] = s_cnt[0] + s_cnt[1];
         p.cls[row] = kClsBmrWide;
@@ -1041,6 +1073,7 @@ __global__ void __launch_bounds__(kPlanThreads, 16) bmr_plan_kernel(const RowPla
       prod += static_cast<unsigned long long>(hr.y);
     }
   }
+  if (clr_pending && !mbar_wait(&s_mbar, mphase) && t == 0) atomicOr(&p.sum->status, kErrCount);
   if (t == 0) {
     if (taken) atomicAdd(&p.sum->seg_count[kSegBmrWide], taken);
     if (prod) atomicAdd(reinterpret_cast<unsigned long long*>(&p.sum->products), prod);
