@@ -755,7 +755,7 @@ def run_ours(args, world, rank, local, pg) -> None:
         if rank == 0:
             sustained = {"steps": sus["steps"], "ms_per_step": sus["ms_per_step"], "value": sus["value"],
                          "unit": sus["unit"], "timed_region_s": round(sus["_total_s"], 3), "clocks": sus["clocks"]}
-    # Every named SpGEMM workload (BASELINE's five configurations), on a single GPU.
+    # Every named SpGEMM workload (the five configurations of the headline metric), on a single GPU.
     per_config = None
     if args.per_config and not ew and not args.rows and world == 1:
         per_config = {}
