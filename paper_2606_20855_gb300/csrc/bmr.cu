@@ -13,8 +13,9 @@
 // Numeric pass.  No workspace search is left: the first product of every
 // column stores its column and value at its stored rank in a compact staging
 // array, the products that repeat a column then add theirs (a shared-memory
-// atomic, the atomic level of Sec. 4), and the warp copies the sorted row to
-// C with coalesced stores.  One warp owns the row (shard pattern, Sec. 4).
+// atomic, the atomic level of Sec. 4), and the sorted row leaves the staging
+// for C (a bulk copy for long rows, coalesced lane stores otherwise).  One
+// warp owns the row (shard pattern, Sec. 4).
 //
 // Lanes are split into groups of G lanes; the group of lane l takes stored A
 // entries j = l / G, l / G + 32/G, ...; lane l takes element l % G of B[k_j,:].
@@ -28,9 +29,10 @@
 //
 // Planning.  When B has at most 65,536 columns every row fits a bitmap over
 // all columns (lo = 0), and bmr_plan_kernel ranks every eligible row of A in
-// the first pass over A, two warps per row (no separate analysis pass for
-// those rows); the rows it does not take are queued for the analysis kernel.
-// Its numeric pass is bmr_numeric_kernel, as for the binned rows.
+// the first pass over A, a CTA of two warps per row (no separate analysis
+// pass for those rows); the rows it does not take are queued for the
+// analysis kernel.  Its numeric pass is bmr_numeric_kernel, as for the
+// binned rows.
 #include <climits>
 #include <type_traits>
 

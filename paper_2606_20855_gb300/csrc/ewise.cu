@@ -30,7 +30,9 @@
 // (chunk output offsets, nnz(C)) -> C.rowptr[i] = offset of the first chunk
 // of row i (of the next chunk for an empty row).  Numeric pass: every chunk
 // reads its split and the next chunk's, merges again and writes its entries
-// from its offset.
+// from its offset.  The default for short rows merges one chunk per lane
+// from shared-memory copies of a warp's 32 chunks (ew_tile_kernel); its
+// count keeps each chunk's absolute start in A and B instead of the split.
 #include <climits>
 
 #include "ws_internal.cuh"
