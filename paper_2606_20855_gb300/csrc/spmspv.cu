@@ -65,16 +65,31 @@ __device__ __forceinline__ int64_t warp_last_le(const int64_t* off, int64_t lo, 
 // warps find the x entries holding the first and the last, the offsets of
 // that range go to shared memory (when it fits), and every thread finds the
 // entry of each of its products by binary search there.
+// Positions of y below kPrivRows are summed in a CTA-private copy in shared
+// memory and added to y once per CTA at the end: adds to one address of y
+// serialise in L2, and a power-law matrix concentrates its products on a few
+// rows (an R-MAT matrix without vertex permutation on its first rows).  The
+// result is the same for any input; only the speed depends on where the
+// heavy rows lie.
 constexpr int kPerThread = 8;
 constexpr int kScatterTile = kSvThreads * kPerThread;
 constexpr int kScatterSpan = 2048;  // x entries of one tile kept in shared memory
+constexpr int kPrivRows = 4096;     // positions of y summed per CTA in shared memory first
 
 template <typename T>
 __global__ void __launch_bounds__(kSvThreads) sv_scatter_kernel(const SpmspvPlan<T> p) {
   __shared__ long long s_off[kScatterSpan + 1];
   __shared__ long long s_k[2];
+  __shared__ T s_acc[kPrivRows];
+  __shared__ uint8_t s_hit[kPrivRows];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t total = p.off[p.nx];
+  const int priv = static_cast<int>(p.m < kPrivRows ? p.m : kPrivRows);
+  for (int i = threadIdx.x; i < kPrivRows; i += blockDim.x) {
+    s_acc[i] = T(0);
+    s_hit[i] = 0;
+  }
+  __syncthreads();
   bool bad = false;
   for (int64_t t0 = static_cast<int64_t>(blockIdx.x) * kScatterTile; t0 < total;
        t0 += static_cast<int64_t>(gridDim.x) * kScatterTile) {
@@ -152,10 +167,22 @@ __global__ void __launch_bounds__(kSvThreads) sv_scatter_kernel(const SpmspvPlan
         bad = true;
         continue;
       }
-      atomicAdd(p.acc + i, vv[r]);
-      p.mark[i] = 1;
+      if (i < priv) {
+        atomicAdd(s_acc + i, vv[r]);
+        s_hit[i] = 1;
+      } else {
+        atomicAdd(p.acc + i, vv[r]);
+        p.mark[i] = 1;
+      }
     }
     __syncthreads();  // s_off and s_k are reused by the next tile
+  }
+  // The CTA's private sums: one add per position it hit.
+  for (int i = threadIdx.x; i < priv; i += blockDim.x) {
+    if (s_hit[i]) {
+      atomicAdd(p.acc + i, s_acc[i]);
+      p.mark[i] = 1;
+    }
   }
   if (bad) atomicOr(&p.sum->status, kErrCount);
 }
