@@ -291,6 +291,44 @@ def test_wide_heavy_rows(dtype):
     assert_matches_oracle(A, B, rowptr, colidx, vals)
 
 
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_wide_rows_cluster_split(dtype):
+    """Wide-bitmap rows whose column ranges sit at the edges of the split of a
+    row's bitmap over a cluster of CTAs (runs of a power of two of 128-column
+    chunks): one chunk (spans 1 and 128), one chunk past a power of two,
+    ranges that leave some CTAs of the cluster without a chunk, the full
+    2^20 columns, and one row of many stored entries in the same kernel."""
+    rng = np.random.default_rng(33)
+    n = 1 << 20
+    spans = [1, 127, 128, 129, 1024, 1025, 65537, (1 << 19) + 1, (1 << 20) - 5, 1 << 20]
+    b_rows, a_rows = [], {}
+    for i, s in enumerate(spans):
+        c0 = int(rng.integers(0, n - s + 1))
+        first = len(b_rows)
+        for j in range(40):
+            cols = set(int(c) for c in c0 + rng.integers(0, s, size=int(rng.integers(1, 9))))
+            if j == 0:
+                cols.add(c0)            # the row's range is exactly [c0, c0 + s)
+            if j == 39:
+                cols.add(c0 + s - 1)
+            b_rows.append(sorted(cols))
+        a_rows[i] = list(range(first, first + 40))
+    hub = len(spans)  # many stored entries over rows spanning all columns
+    first = len(b_rows)
+    for j in range(3000):
+        b_rows.append(sorted(set(int(c) for c in rng.integers(0, n, size=5))))
+    a_rows[hub] = list(range(first, first + 3000))
+    B = _csr(len(b_rows), n, dict(enumerate(b_rows)), dtype=dtype)
+    B.vals = (1.0 - rng.random(B.nnz)).astype(dtype)
+    A = _csr(len(spans) + 1, B.nrows, a_rows, dtype=dtype)
+    A.vals = (2 * rng.random(A.nnz) - 1).astype(dtype)
+    with tuning(hash_max_products=0, bitmap_span=0, dense_rows_max_a=0, register_rows_max_a=0):
+        rowptr, colidx, vals, info = run_gpu(A, B)
+    assert info["wb_rows"] == len(spans) + 1
+    assert_matches_oracle(A, B, rowptr, colidx, vals)
+    assert rowptr[1] == 1  # span 1: forty products, one column
+
+
 @pytest.mark.parametrize("path", list(PATHS))
 def test_skewed_rmat_square(path):
     rng = np.random.default_rng(14)
